@@ -1,0 +1,383 @@
+"""Pins for the oracle (CPU only).
+
+Each test ties the oracle to something other than itself: a closed form the
+paper prints (App. A, Sec. 3.2), a textbook identity worked by hand (fixtures
+under tests/golden/), a library routine on a special case (numpy polynomial
+and linear-algebra routines, torch's fp32->bf16 conversion), or brute force on
+small inputs. The last group plants mistakes in copies of the oracle's weights
+and checks that the pins catch them.
+"""
+import math
+import os
+from fractions import Fraction
+
+import numpy as np
+import pytest
+
+GOLD = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _rows(name):
+    out = []
+    with open(os.path.join(GOLD, name)) as fh:
+        for line in fh:
+            line = line.strip()
+            if not line or line.startswith("#"):
+                continue
+            lhs, rhs = line.split(":")
+            out.append((lhs.split(), rhs.split()))
+    return out
+
+
+def _rel(a, b):
+    a, b = np.asarray(a, np.float64), np.asarray(b, np.float64)
+    return float(np.max(np.abs(a - b)) / max(np.max(np.abs(b)), 1e-300))
+
+
+# ------------------------------------------------------------------ bf16 codec
+def test_bf16_golden(orc):
+    for lhs, rhs in _rows("bf16_encodings.txt"):
+        x = float.fromhex(lhs[0])
+        assert int(orc.bf16_encode([x])[0]) == int(rhs[0], 16), (lhs, rhs)
+
+
+def _bf16_table():
+    bits = np.arange(0x7F80, dtype=np.uint32)  # +0 .. largest finite
+    vals = (bits << 16).view(np.float32).astype(np.float64)
+    return bits.astype(np.int64), vals
+
+
+def _bf16_bruteforce(x, bits, vals):
+    """Nearest finite bf16 by exhaustive search, ties to the even pattern."""
+    a = abs(x)
+    sign = 0x8000 if math.copysign(1.0, x) < 0 else 0
+    top = vals[-1]
+    half_ulp_top = (vals[-1] - vals[-2]) / 2
+    if Fraction(a) >= Fraction(top) + Fraction(half_ulp_top):
+        return sign | 0x7F80
+    i = int(np.searchsorted(vals, a))
+    cands = [k for k in (i - 1, i, i + 1) if 0 <= k < len(vals)]
+    fa = Fraction(a)
+    best = min(abs(Fraction(vals[k]) - fa) for k in cands)
+    ties = [k for k in cands if abs(Fraction(vals[k]) - fa) == best]
+    k = ties[0] if len(ties) == 1 else [t for t in ties if bits[t] % 2 == 0][0]
+    return sign | int(bits[k])
+
+
+def test_bf16_bruteforce_nearest(orc):
+    rng = np.random.default_rng(2025)
+    bits, vals = _bf16_table()
+    xs = list(rng.uniform(0.5, 1.0, 300) * np.exp2(rng.integers(-140, 129, 300)))
+    xs = [x * (-1 if rng.random() < 0.5 else 1) for x in xs]
+    # exact midpoints between neighbouring bf16 values, and their neighbours
+    ks = rng.integers(0, len(vals) - 1, 200)
+    for k in ks:
+        m = (vals[k] + vals[k + 1]) / 2  # exact in fp64 (9 significant bits)
+        xs += [m, np.nextafter(m, 0.0), np.nextafter(m, np.inf)]
+    xs += [5e-324, 1e-45, 3e38, 3.4e38, 3.3961e38, 1e300]
+    for x in xs:
+        assert int(orc.bf16_encode([x])[0]) == _bf16_bruteforce(float(x), bits, vals), float(x).hex()
+
+
+def test_bf16_matches_torch_on_fp32_inputs(orc):
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(7)
+    raw = rng.integers(0, 2**32, 20000, dtype=np.uint64).astype(np.uint32)
+    f = raw.view(np.float32)
+    f = f[np.isfinite(f)]
+    # one rounding from fp32 is the same as one rounding from its exact fp64 value
+    ref = torch.from_numpy(f.copy()).to(torch.bfloat16).view(torch.int16).numpy().astype(np.uint16)
+    got = orc.bf16_encode(f.astype(np.float64))
+    assert np.array_equal(got, ref)
+
+
+def test_bf16_decode_all_patterns(orc):
+    h = np.arange(65536, dtype=np.uint32)
+    finite = ((h >> 7) & 0xFF) != 0xFF
+    h = h[finite].astype(np.uint16)
+    ref = (h.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    dec = orc.bf16_decode(h)
+    assert np.array_equal(dec, ref)
+    assert np.array_equal(orc.bf16_encode(dec), h)  # every bf16 value round-trips
+
+
+# -------------------------------------------------------------------- schedule
+def test_full_schedule_golden(orc):
+    for lhs, rhs in _rows("full_schedule.txt"):
+        T, r, s0, s1, K = map(int, lhs)
+        mask = orc.full_schedule(T, r, s0, s1, K)
+        if rhs[0].startswith("#"):
+            assert int(mask.sum()) == int(rhs[0][1:]), lhs
+        else:
+            assert list(np.nonzero(mask)[0]) == [int(v) for v in rhs], lhs
+
+
+def test_normalize_endpoints(orc):
+    tau = orc.normalize([0.0, 999.0, 499.5, 249.75], 0.0, 999.0)
+    assert list(tau) == [-1.0, 1.0, 0.0, -0.5]
+
+
+# --------------------------------------------------------------------- weights
+def test_rho_equispaced_closed_form(orc):
+    for lhs, rhs in _rows("equispaced_rho.txt"):
+        N = int(lhs[0])
+        x = np.array([-1 + 2 * (j - 1) / (N - 1) for j in range(1, N + 1)])
+        r = orc.rho(x)
+        g = np.array([float(v) for v in rhs])
+        assert _rel(r / r[0], g / g[0]) <= 1e-14, N
+
+
+def test_rho_chebyshev_extrema_printed_form(orc):
+    for lhs, rhs in _rows("chebyshev_extrema_rho.txt"):
+        N = int(lhs[0])
+        x = np.cos(np.arange(N) * np.pi / (N - 1))
+        r = orc.rho(x)
+        g = np.array([float(v) for v in rhs])
+        assert _rel(r / r[0], g / g[0]) <= 1e-13, N
+
+
+def test_rho_chebyshev_roots(orc):
+    """Roots of T_N (Sec. 3.2 node formula). Their weights are
+    (-1)^j sin((2j-1) pi / (2N)) (Berrut & Trefethen, SIAM Review 2004), which
+    differ from the printed extrema form whenever N >= 4 (for N = 3 both
+    reduce to (-1/2, 1, -1/2) up to sign)."""
+    _, extrema = zip(*_rows("chebyshev_extrema_rho.txt"))
+    for N in range(2, 9):
+        j = np.arange(1, N + 1)
+        x = np.cos((2 * j - 1) * np.pi / (2 * N))
+        r = orc.rho(x)
+        g = (-1.0) ** j * np.sin((2 * j - 1) * np.pi / (2 * N))
+        assert _rel(r / r[0], g / g[0]) <= 1e-13, N
+        if N >= 4:
+            pe = np.array([float(v) for v in extrema[N - 2]])
+            assert _rel(r / r[0], pe / pe[0]) > 1e-3
+
+
+def test_weights_golden(orc):
+    for lhs, rhs in _rows("extrapolation_weights.txt"):
+        N, xq = int(lhs[0]), float(lhs[1])
+        g = np.array([float(v) for v in rhs])
+        nodes = np.arange(N, dtype=np.float64)
+        assert _rel(orc.bary_coeff(nodes, xq), g) <= 1e-13, lhs
+        assert _rel(orc.lagrange_basis(nodes, xq), g) <= 1e-13, lhs
+        # the same nodes mapped onto [-1, 1] (Sec. 3.3 normalisation)
+        lo, hi = 0.0, max(N - 1, 1)
+        tau = orc.normalize(nodes, lo, hi)
+        tq = orc.normalize([xq], lo, hi)[0]
+        assert _rel(orc.lagrange_basis(tau, tq), g) <= 1e-13, lhs
+
+
+def _random_nodes(rng, K):
+    while True:
+        x = np.sort(rng.uniform(-1, 1, K))
+        if K == 1 or np.min(np.diff(x)) > 0.05:
+            return x
+
+
+def test_partition_of_unity(orc):
+    rng = np.random.default_rng(11)
+    for _ in range(300):
+        K = int(rng.integers(1, 9))
+        x = _random_nodes(rng, K)
+        xq = float(rng.uniform(-3, 3))
+        for w in (orc.lagrange_basis(x, xq), orc.bary_coeff(x, xq)):
+            assert abs(w.sum() - 1.0) <= 16 * np.finfo(float).eps * np.abs(w).sum()
+
+
+def test_polynomial_exactness(orc):
+    P = np.polynomial.polynomial
+    rng = np.random.default_rng(12)
+    for _ in range(300):
+        K = int(rng.integers(1, 9))
+        x = _random_nodes(rng, K)
+        xq = float(rng.uniform(-2.5, 2.5))
+        c = rng.standard_normal(K)  # degree <= K-1
+        fx = P.polyval(x, c)
+        w = orc.lagrange_basis(x, xq)
+        scale = np.abs(w * fx).sum() + abs(P.polyval(xq, c))
+        assert abs(w @ fx - P.polyval(xq, c)) <= 1e-10 * scale
+
+
+def test_weights_solve_moment_system(orc):
+    """Brute force: the weights are the unique solution of sum_j w_j x_j^m = x^m,
+    m < K (numpy.linalg.solve on the transposed Vandermonde matrix)."""
+    rng = np.random.default_rng(13)
+    for _ in range(200):
+        K = int(rng.integers(1, 7))
+        x = _random_nodes(rng, K)
+        xq = float(rng.uniform(-2, 2))
+        V = np.vander(x, K, increasing=True)  # V[j, m] = x_j^m
+        ref = np.linalg.solve(V.T, xq ** np.arange(K))
+        assert _rel(orc.lagrange_basis(x, xq), ref) <= 1e-9
+        assert _rel(orc.bary_coeff(x, xq), ref) <= 1e-9
+
+
+def test_error_formula_degree_K(orc):
+    """App. A error formula, exact for a degree-K trajectory: with
+    F = sum_{d<=K} c_d T_d, F(x) - P(x) = c_K 2^(K-1) omega(x)."""
+    C = np.polynomial.chebyshev
+    P = np.polynomial.polynomial
+    rng = np.random.default_rng(14)
+    for _ in range(200):
+        K = int(rng.integers(1, 9))
+        x = _random_nodes(rng, K)
+        xq = float(rng.uniform(-2, 2))
+        c = rng.standard_normal(K + 1)
+        w = orc.lagrange_basis(x, xq)
+        err = C.chebval(xq, c) - w @ C.chebval(x, c)
+        omega = P.polyval(xq, P.polyfromroots(x))
+        ref = c[K] * 2.0 ** (K - 1) * omega if K >= 1 else 0.0
+        scale = np.abs(w * C.chebval(x, c)).sum() + abs(C.chebval(xq, c))
+        assert abs(err - ref) <= 1e-10 * scale
+        assert abs(orc.nodal(x, xq) - omega) <= 1e-12 * max(1.0, abs(omega))
+
+
+def test_affine_invariance(orc):
+    rng = np.random.default_rng(15)
+    for _ in range(100):
+        K = int(rng.integers(2, 9))
+        x = _random_nodes(rng, K)
+        xq = float(rng.uniform(-2, 2))
+        a, b = float(rng.uniform(0.1, 500) * rng.choice([-1, 1])), float(rng.uniform(-500, 500))
+        assert _rel(orc.lagrange_basis(a * x + b, a * xq + b), orc.lagrange_basis(x, xq)) <= 1e-9
+
+
+def test_target_on_node_and_duplicates(orc):
+    x = np.array([-1.0, -0.2, 0.5, 0.9])
+    for j in range(4):
+        e = np.zeros(4)
+        e[j] = 1.0
+        assert np.array_equal(orc.bary_coeff(x, x[j]), e)
+        assert np.array_equal(orc.lagrange_basis(x, x[j]), e)
+    with pytest.raises(ValueError):
+        orc.rho([0.1, 0.3, 0.1])
+
+
+def test_history_fifo(orc):
+    H = orc.History(4)
+    for s in range(7):
+        H.push(1000 - 100 * s, s)
+        assert len(H.entries()) == min(s + 1, 4)
+    assert H.full()
+    assert H.times() == [700.0, 600.0, 500.0, 400.0]
+    assert [f for _, f in H.entries()] == [3, 4, 5, 6]
+
+
+# --------------------------------------------------------------- combination
+def test_extrapolate_fp64_matches_einsum(orc):
+    rng = np.random.default_rng(16)
+    for K in (1, 3, 5, 8):
+        F = [rng.standard_normal(1000).astype(np.float32) for _ in range(K)]
+        w = rng.standard_normal(K)
+        (out,), _ = orc.extrapolate([F], w, orc.FP32, orc.FP64)
+        ref = np.einsum("j,jn->n", w, np.array(F, np.float64))
+        bound = 4 * K * np.finfo(float).eps * np.einsum("j,jn->n", np.abs(w), np.abs(np.array(F, np.float64)))
+        assert np.all(np.abs(out - ref) <= bound)
+
+
+def test_extrapolate_rounds_once(orc):
+    rng = np.random.default_rng(17)
+    K = 4
+    F = [orc.bf16_encode(rng.standard_normal(3000)) for _ in range(K)]
+    w = orc.lagrange_basis(np.array([-1, -1 / 3, 1 / 3, 1.0]), 1.4)
+    (o64,), _ = orc.extrapolate([F], w, orc.BF16, orc.FP64)
+    (o16,), _ = orc.extrapolate([F], w, orc.BF16, orc.BF16)
+    (o32,), _ = orc.extrapolate([F], w, orc.BF16, orc.FP32)
+    assert np.array_equal(o16, orc.bf16_encode(o64))
+    assert np.array_equal(o32, o64.astype(np.float32))
+    # the bf16 inputs are decoded exactly
+    ref = np.einsum("j,jn->n", w, np.array([orc.bf16_decode(f) for f in F]))
+    assert np.max(np.abs(o64 - ref)) <= 1e-13 * np.max(np.abs(ref))
+
+
+def test_fused_residual(orc):
+    rng = np.random.default_rng(18)
+    K, nb, n = 3, 3, 2000
+    F = [[rng.standard_normal(n).astype(np.float32) for _ in range(K)] for _ in range(nb)]
+    X = rng.standard_normal(n).astype(np.float32)
+    w = rng.standard_normal(K)
+    outs, res = orc.extrapolate(F, w, orc.FP32, orc.FP64, X=X, x_dtype=orc.FP32, resid_dtype=orc.FP64)
+    Fa = np.array(F, np.float64)  # [nb, K, n]
+    P = np.einsum("j,bjn->bn", w, Fa)
+    assert _rel(np.array(outs), P) <= 1e-14
+    assert _rel(res, X.astype(np.float64) + P.sum(0)) <= 1e-14
+    _, res16 = orc.extrapolate(F, w, orc.FP32, None, X=X, x_dtype=orc.FP32, resid_dtype=orc.BF16)
+    assert np.array_equal(res16, orc.bf16_encode(res))
+
+
+def test_threads_identical(orc):
+    rng = np.random.default_rng(19)
+    F = [orc.bf16_encode(rng.standard_normal(10001)) for _ in range(5)]
+    w = rng.standard_normal(5)
+    (a,), _ = orc.extrapolate([F], w, orc.BF16, orc.BF16, nthreads=1)
+    (b,), _ = orc.extrapolate([F], w, orc.BF16, orc.BF16, nthreads=7)
+    assert np.array_equal(a, b)
+
+
+def test_convert_matches_torch(orc):
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(20)
+    f = np.concatenate([rng.standard_normal(5000).astype(np.float32),
+                        np.array([1e-40, -3e-39, 3.39e38, -0.0, 0.0], np.float32)])
+    ref = torch.from_numpy(f).to(torch.bfloat16).view(torch.int16).numpy().astype(np.uint16)
+    assert np.array_equal(orc.convert(f, orc.FP32, orc.BF16), ref)
+    h = rng.integers(0, 65536, 5000).astype(np.uint16)
+    assert np.array_equal(orc.convert(h, orc.BF16, orc.BF16), h)  # bit copy, NaN patterns too
+    assert np.array_equal(orc.convert(f, orc.FP32, orc.FP32), f)
+
+
+# ------------------------------------------------------- planted mistakes
+def _weight_pins(fn, orc):
+    """Run the weight pins against ``fn(x, xq)``; return the names that fail."""
+    failed = set()
+    rng = np.random.default_rng(21)
+    C = np.polynomial.chebyshev
+    P = np.polynomial.polynomial
+    for lhs, rhs in _rows("extrapolation_weights.txt"):
+        N, xq = int(lhs[0]), float(lhs[1])
+        if _rel(fn(np.arange(N, dtype=float), xq), np.array([float(v) for v in rhs])) > 1e-12:
+            failed.add("golden")
+    for _ in range(50):
+        K = int(rng.integers(2, 7))
+        x = _random_nodes(rng, K)
+        xq = float(rng.uniform(1.05, 2))
+        w = fn(x, xq)
+        if abs(w.sum() - 1) > 1e-12 * np.abs(w).sum():
+            failed.add("unity")
+        c = rng.standard_normal(K)
+        if abs(w @ P.polyval(x, c) - P.polyval(xq, c)) > 1e-9 * (np.abs(w).sum() + 1) * np.abs(c).sum():
+            failed.add("exact")
+        c = rng.standard_normal(K + 1)
+        err = C.chebval(xq, c) - w @ C.chebval(x, c)
+        ref = c[K] * 2.0 ** (K - 1) * P.polyval(xq, P.polyfromroots(x))
+        if abs(err - ref) > 1e-9 * (np.abs(w).sum() + 1) * np.abs(c).sum() * 4:
+            failed.add("error-formula")
+    return failed
+
+
+def test_pins_catch_planted_mistakes(orc):
+    good = lambda x, xq: orc.lagrange_basis(x, xq)
+    assert _weight_pins(good, orc) == set()
+
+    def sign_flip(x, xq):
+        w = good(x, xq).copy()
+        w[1] = -w[1]
+        return w
+
+    def reversed_order(x, xq):  # weights paired with the wrong history entries
+        return good(x, xq)[::-1].copy()
+
+    def dropped_node(x, xq):  # rho from all but the oldest node
+        w = np.zeros(len(x))
+        w[1:] = good(x[1:], xq) if len(x) > 1 else 1.0
+        return w
+
+    def wrong_target(x, xq):  # target mapped with an off-by-one-spacing error
+        return good(x, xq + (x[-1] - x[-2]))
+
+    def no_normalisation(x, xq):  # first barycentric form without the omega factor
+        r = orc.rho(x)
+        return r / (xq - x)
+
+    for bad in (sign_flip, reversed_order, dropped_node, wrong_target, no_normalisation):
+        assert _weight_pins(bad, orc), bad.__name__
