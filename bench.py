@@ -1,0 +1,417 @@
+"""Benchmark of the skipped-step extrapolation (Sec. 3.3, Eq. for f_t) on GB300.
+
+One step = one skipped diffusion step over every block of the workload: the
+host computes the fp64 weights for the target timestep from the live history
+and one grouped persistent kernel streams the K cached slots of every branch
+tensor and writes the predictions (HBM-bound K-term reduction).
+
+Default workload: FLUX.1-dev 1024^2 shapes (19 double-stream blocks with image
+and text streams, 38 single-stream blocks: 114 bf16 tensors, 1.08 G elements
+per slot, K = 5). The history is filled by walking the 50-step schedule
+(r = 6) to a mid-schedule window of K equispaced nodes; the timed steps cycle
+over that window's skipped targets. Inputs (12.9 GB per step) exceed L2
+(~129 MB), so no flush is needed between steps.
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME]
+                       [--impl ours|reference]
+Under torchrun each rank runs its own replica (independent samples, no data
+exchange); timing is the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "extrapolation GB/s & % of HBM peak; µs per skipped step (all blocks), 1 GB300"
+KERNEL_SOURCES = ["paper_2608_23429_gb300/csrc/extrapolate.cu", "paper_2608_23429_gb300/csrc/cb_device.h"]
+
+
+def kernel_hash() -> str:
+    h = hashlib.sha256()
+    for p in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, p), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def measured_peaks() -> tuple[float, str]:
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as fh:
+            return float(json.load(fh)["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, "fallback"
+
+
+def recorded_traffic(config: str) -> float | None:
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on
+    the current kernel source (else None)."""
+    path = os.path.join(ROOT, "profiles", f"extrapolate_{config}_traffic.txt")
+    try:
+        fields = dict(line.split("=", 1) for line in open(path).read().split() if "=" in line)
+    except OSError:
+        return None
+    if fields.get("kernel_sha") != kernel_hash():
+        return None
+    try:
+        return float(fields["dram_bytes_per_launch"])
+    except (KeyError, ValueError):
+        return None
+
+
+class Clocks:
+    """nvidia-smi sampling during the timed region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        self.p = None
+
+    def __enter__(self):
+        try:
+            self.p = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                                       "--format=csv,noheader,nounits", "-lms", "200"],
+                                      stdout=self.f, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.p = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        if self.p is not None:
+            self.p.terminate()
+            try:
+                self.p.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.p.kill()
+
+    def summary(self) -> dict:
+        self.f.flush()
+        rows = []
+        for line in open(self.f.name).read().splitlines():
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append(dict(sm=float(parts[1]), max=float(parts[2]), power=float(parts[3]),
+                                 hw=parts[5], hwt=parts[6], swt=parts[7], swp=parts[8]))
+            except ValueError:
+                continue
+        os.unlink(self.f.name)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"], "samples": 0}
+        top = max(r["power"] for r in rows)
+        load = [r for r in rows if r["power"] >= 0.5 * top] or rows
+        reasons = []
+        for key, name in (("hw", "hw_slowdown"), ("hwt", "hw_thermal_slowdown"),
+                          ("swt", "sw_thermal_slowdown"), ("swp", "sw_power_cap")):
+            if any(r[key].lower().startswith("active") for r in load):
+                reasons.append(name)
+        return {"sm_mhz": statistics.median(r["sm"] for r in load), "sm_max_mhz": max(r["max"] for r in rows),
+                "reasons": reasons, "samples": len(load), "power_w_max": top}
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def max_over_ranks(x: float, device) -> float:
+    """Max of a per-rank timing over all ranks (measurement only; no data moves)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return x
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def workload_description(w) -> dict:
+    slot = sum(t.numel for t in w.tensors) * w.esize()
+    return {"workload": w.name, "tensors": len(w.tensors), "K": w.K, "storage": w.cache_dtype,
+            "slot_bytes": slot, "schedule": f"T={w.T}, full every r={w.r}"}
+
+
+def pick_window(w, orc):
+    """Walk the schedule to the first window of K equispaced nodes past the
+    warm-up; return (full steps pushed in order, skipped steps that follow)."""
+    mask = orc.full_schedule(w.T, w.r, w.s0, w.s1, w.K)
+    full = [s for s in range(w.T) if mask[s]]
+    for k in range(w.K - 1, len(full) - 1):
+        win = full[k - w.K + 1:k + 1]
+        if len({b - a for a, b in zip(win, win[1:])}) == 1 and win[-1] - win[0] == w.r * (w.K - 1):
+            targets = [s for s in range(win[-1] + 1, full[k + 1])]
+            if targets:
+                return full[:k + 1], targets
+    raise RuntimeError("no equispaced window in the schedule")
+
+
+def cpu_oracle_run(w, feats_host, wts, seconds: float, nthreads: int):
+    """Time the oracle on a bounded sample; returns (GB/s, elements, reps, seconds)."""
+    import oracle as orc
+    reps, t0 = 0, time.perf_counter()
+    n = feats_host[0].size
+    while True:
+        orc.extrapolate([feats_host], wts, orc.BF16, orc.BF16, nthreads=nthreads)
+        reps += 1
+        el = time.perf_counter() - t0
+        if el >= seconds:
+            break
+    gbs = reps * n * (w.K + 1) * 2 / el / 1e9
+    return gbs, n, reps, el
+
+
+def sample_host_features(w, torch, wl, orc, n_elems: int, device):
+    """A bounded contiguous sample of the largest tensor at K nodes (generator bytes)."""
+    i = max(range(len(w.tensors)), key=lambda k: w.tensors[k].numel)
+    _, targets = pick_window(w, orc)
+    full, _ = pick_window(w, orc)
+    nodes = full[-w.K:]
+    host = []
+    for s in nodes:
+        f = wl.trajectory(w, i, w.timesteps[s], s, device).reshape(-1)[:n_elems]
+        host.append(f.contiguous().cpu().view(torch.int16).numpy().view("uint16").copy())
+    t_nodes = [w.timesteps[s] for s in nodes]
+    wts = orc.weights(t_nodes, w.timesteps[targets[0]], w.t_min, w.t_max)
+    return host, wts, i
+
+
+def run_reference(args):
+    """The oracle on the host cores: each step is a bounded sample of the workload."""
+    ws, rank, _ = dist_env()
+    if rank != 0:
+        return 0
+    import numpy as np
+    import torch
+
+    import oracle as orc
+    from paper_2608_23429_gb300 import workloads as wl
+    orc.build()
+    w = wl.PRESETS[args.config]()
+    n = args.cpu_elems
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    host, wts, ti = sample_host_features(w, torch, wl, orc, n, dev)
+    threads = os.cpu_count() or 1
+    for _ in range(args.warmup):
+        orc.extrapolate([host], wts, orc.BF16, orc.BF16, nthreads=threads)
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        orc.extrapolate([host], wts, orc.BF16, orc.BF16, nthreads=threads)
+        times.append(time.perf_counter() - t0)
+    total = sum(times)
+    bytes_step = n * (w.K + 1) * 2
+    value = bytes_step * args.steps / total / 1e9
+    desc = workload_description(w)
+    sample = f"{n} contiguous elements of tensor {ti} (K={w.K} bf16 slots + bf16 output) per step"
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": "GB/s", "n_gpus": ws,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(total / args.steps * 1e3, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": dict(desc, sample=sample),
+        "cpu_baseline": {"value": round(value, 3), "unit": "GB/s", "cores": threads, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": round(value, 3), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    del np
+    return 0
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    ws, rank, local = dist_env()
+    if ws > 1:
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", init_method="env://")
+    else:
+        torch.cuda.set_device(0)
+    dev = torch.device("cuda", torch.cuda.current_device())
+
+    import oracle as orc
+    from paper_2608_23429_gb300 import build as cbuild
+    cbuild.build()
+    orc.build()
+    from paper_2608_23429_gb300 import chebboost as cb
+    from paper_2608_23429_gb300 import workloads as wl
+
+    w = wl.PRESETS[args.config]()
+    if args.scale > 1:
+        w = wl.scaled(w, args.scale)
+    K = w.K
+    pushed, targets = pick_window(w, orc)
+    node_t = [w.timesteps[s] for s in orc.full_schedule(w.T, w.r, w.s0, w.s1, K).nonzero()[0]]
+    tensors = [(t.layer, t.branch, t.numel, t.group) for t in w.tensors]
+    cdt = cb.CB_BF16 if w.cache_dtype == "bf16" else cb.CB_FP32
+    tdt = torch.bfloat16 if w.cache_dtype == "bf16" else torch.float32
+    plan = cb.cb_plan_create(node_t, K, tensors, cdt, w.t_min, w.t_max)
+    cache = torch.empty(cb.cb_plan_cache_bytes(plan), dtype=torch.uint8, device=dev)
+    cb.cb_plan_bind_cache(plan, cache, cache.numel())
+    stream = torch.cuda.Stream(device=dev)
+    for s in pushed:  # full steps of the schedule up to the timed window
+        feats = [wl.trajectory(w, i, w.timesteps[s], s, dev) for i in range(len(w.tensors))]
+        torch.cuda.synchronize()
+        cb.cb_cache_push(plan, feats, cdt, w.timesteps[s], stream=stream)
+        stream.synchronize()
+        del feats
+    outs = [torch.empty(t.shape, dtype=tdt, device=dev) for t in w.tensors]
+    slot_elems = sum(t.numel for t in w.tensors)
+    esz = 2 if w.cache_dtype == "bf16" else 4
+    bytes_step = slot_elems * esz * (K + 1)  # K slot reads + one output write
+    t_targets = [w.timesteps[s] for s in targets]
+
+    def step(k):
+        cb.cb_extrapolate(plan, t_targets[k % len(t_targets)], outs, cdt, stream=stream)
+
+    for k in range(args.warmup):
+        step(k)
+    stream.synchronize()
+    if ws > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    with Clocks(torch.cuda.current_device()) as clk:
+        t_all0 = torch.cuda.Event(enable_timing=True)
+        t_all1 = torch.cuda.Event(enable_timing=True)
+        t_all0.record(stream)
+        for k in range(args.steps):
+            ev[k][0].record(stream)
+            step(k)
+            ev[k][1].record(stream)
+        t_all1.record(stream)
+        stream.synchronize()
+        torch.cuda.synchronize()
+        if ws > 1:
+            dist.barrier()
+    clocks = clk.summary()
+    total_ms = t_all0.elapsed_time(t_all1)
+    kern_ms = [a.elapsed_time(b) for a, b in ev]
+    total_ms = max_over_ranks(total_ms, dev)
+    ms_step = total_ms / args.steps
+    value = bytes_step * args.steps * ws / (total_ms / 1e3) / 1e9
+    avg_kern = sum(kern_ms) / len(kern_ms)
+    peak, peak_src = measured_peaks()
+    achieved = bytes_step / (avg_kern / 1e3) / 1e9
+
+    # ---- end to end through the public API with host buffers: upload the K
+    # cached feature sets from pinned host memory (push), extrapolate, read the
+    # predictions back; every copy is inside the timed region.
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(args, torch, cb, wl, w, plan, cdt, tdt, dev, pushed, t_targets, bytes_step, ws)
+
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu:
+        host, wts, ti = sample_host_features(w, torch, wl, orc, args.cpu_elems, dev)
+        threads = os.cpu_count() or 1
+        gbs, n, reps, el = cpu_oracle_run(w, host, wts, args.cpu_seconds, threads)
+        cpu = {"value": round(gbs, 3), "unit": "GB/s", "cores": threads, "kind": "oracle",
+               "sample": f"{n} contiguous elements of tensor {ti} at the first timed target, "
+                         f"{reps} passes in {el:.1f} s (fp64 oracle, bf16 in/out)"}
+
+    cb.cb_plan_destroy(plan)
+    if rank == 0:
+        desc = workload_description(w)
+        desc.update({"bytes_per_step": bytes_step, "targets": targets, "history_steps": pushed[-K:],
+                     "l2": "inputs larger than L2 (no flush)", "launch": "1 grouped persistent kernel per step",
+                     "parallelism": f"replicas x{ws}" if ws > 1 else "1 GPU"})
+        line = {
+            "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": ws, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(ms_step, 4),
+            "us_per_step": round(ms_step * 1e3, 2), "pct_hbm_peak": round(100 * value / ws / peak, 2),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic", "config": desc,
+            "roofline": {"bound": "hbm", "achieved": round(achieved, 2), "peak": peak, "unit": "GB/s",
+                         "frac": round(achieved / peak, 4), "peak_source": peak_src,
+                         "traffic": recorded_traffic(args.config) if args.scale == 1 else None,
+                         "kernel": "extrapolate_kernel", "avg_launch_us": round(avg_kern * 1e3, 2)},
+            "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks, "gpu_launches": args.steps,
+        }
+        print(json.dumps(line))
+    if ws > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def run_e2e(args, torch, cb, wl, w, plan, cdt, tdt, dev, pushed, t_targets, bytes_step, ws):
+    K = w.K
+    nodes = pushed[-K:]
+    host_feats = []  # K sets of pinned host features (the full steps' outputs)
+    for s in nodes:
+        host_feats.append([wl.trajectory(w, i, w.timesteps[s], s, dev).cpu().pin_memory()
+                           for i in range(len(w.tensors))])
+    dev_feats = [torch.empty(t.shape, dtype=tdt, device=dev) for t in w.tensors]
+    outs = [torch.empty(t.shape, dtype=tdt, device=dev) for t in w.tensors]
+    host_outs = [torch.empty(t.shape, dtype=tdt).pin_memory() for t in w.tensors]
+    stream = torch.cuda.Stream(device=dev)
+    slot = sum(t.numel for t in w.tensors) * (2 if w.cache_dtype == "bf16" else 4)
+
+    def step(k):
+        cb.cb_plan_reset(plan)
+        with torch.cuda.stream(stream):
+            for j, s in enumerate(nodes):
+                for d, h in zip(dev_feats, host_feats[j]):
+                    d.copy_(h, non_blocking=True)
+                cb.cb_cache_push(plan, dev_feats, cdt, w.timesteps[s], stream=stream)
+            cb.cb_extrapolate(plan, t_targets[k % len(t_targets)], outs, cdt, stream=stream)
+            for h, o in zip(host_outs, outs):
+                h.copy_(o, non_blocking=True)
+
+    steps = max(1, args.e2e_steps)
+    for k in range(2):
+        step(k)
+    stream.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for k in range(steps):
+        step(k)
+    b.record(stream)
+    stream.synchronize()
+    ms = max_over_ranks(a.elapsed_time(b) / steps, dev)
+    return {"value": round(bytes_step * ws / (ms / 1e3) / 1e9, 2), "unit": "GB/s",
+            "h2d_bytes_per_step": K * slot, "d2h_bytes_per_step": slot, "ms_per_step": round(ms, 3),
+            "steps": steps}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--config", default="flux", choices=["dit256", "dit256-k3", "dit512", "pixart", "flux"])
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--scale", type=int, default=1,
+                    help="divide every tensor's token count (small cases for profiling only)")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--cpu-elems", type=int, default=1 << 24)
+    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

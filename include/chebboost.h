@@ -1,0 +1,192 @@
+/*
+ * chebboost.h — C ABI of libchebboost, a GB300 (sm_103a) implementation of the
+ * online extrapolation stage of ChebBooster (training-free DiT acceleration by
+ * Chebyshev-inspired barycentric extrapolation).
+ *
+ * The method (paper Sec. 3.2-3.3, Alg. 1):
+ *   - on full-computation steps s in F, every block's branch outputs f_s are
+ *     stored in a history buffer H that holds the n = K most recent
+ *     (s_j, f_j) pairs, dropping the oldest (Sec. 3.3, "ChebBooster Forward
+ *     Application"; Alg. 1, full-computation branch);
+ *   - on every other step t the features are predicted as
+ *         f_t = sum_j w^j_t f_{s_j}                       (Sec. 3.3, Eq. for f_t)
+ *     with the barycentric interpolation coefficients
+ *         w^j_t = (rho_j / (tau - tau_j)) / sum_i rho_i / (tau - tau_i)
+ *                                                  (Sec. 3.2, Eq. barycentric_coeff)
+ *     where rho_j = 1 / prod_{k != j} (tau_j - tau_k)   (App. A, Eq. general_weights)
+ *     and tau is the timestep mapped affinely onto [-1, 1] (Sec. 3.3).
+ *
+ * Conventions for every call:
+ *   - Host/device: "device pointer" means memory of the current CUDA device;
+ *     "host pointer" means ordinary process memory. The plan holds host state
+ *     only; the caller owns and allocates every device buffer (cache arena,
+ *     features, outputs, hidden states) and every stream.
+ *   - Streams: `stream` is a cudaStream_t passed as void* (NULL = the legacy
+ *     default stream). Device work is enqueued on it asynchronously; no call
+ *     synchronises the device.
+ *   - Errors: every call validates all of its arguments before enqueueing
+ *     anything. On a negative status nothing was enqueued and the plan's
+ *     state (its history) is unchanged. CB_ERR_CUDA reports a failed launch;
+ *     cb_last_error_message() gives the CUDA error text.
+ *   - Threads: a plan is not internally locked; calls on the same plan must
+ *     be serialised by the caller. Different plans are independent.
+ *   - Layout: each branch tensor is a contiguous row-major array
+ *     [batch, tokens, hidden] of `numel` elements. Pointers must be aligned to
+ *     their element size; pointers aligned to 16 bytes take the vectorised
+ *     path, others a scalar path (same results).
+ *   - Rounding: fp32 -> bf16 conversions round to nearest, ties to even.
+ */
+#ifndef CHEBBOOST_H
+#define CHEBBOOST_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define CB_MAX_K 8            /* largest history size n (Sec. 3.3) */
+#define CB_MAX_TENSORS 256    /* branch tensors per plan */
+#define CB_MAX_BRANCHES 4     /* branch tensors sharing one residual group */
+#define CB_CACHE_ALIGN 256    /* byte alignment of the cache arena and of each tensor in it */
+
+typedef struct cb_plan cb_plan; /* opaque, host-owned */
+
+typedef enum { CB_BF16 = 0, CB_FP32 = 1 } cb_dtype;
+
+/* One cached branch tensor (Sec. 3.1: the self-attention, cross-attention
+ * and MLP outputs S^l, C^l, M^l of block l). `group` names the hidden state
+ * the branch is added into (B^l(x) = x + S^l + C^l + M^l): tensors with the
+ * same group share one residual pointer in cb_extrapolate and must have the
+ * same numel; -1 means the tensor has no residual. */
+typedef struct {
+    int32_t layer;    /* block index l (informational) */
+    int32_t branch;   /* branch index inside the block (informational) */
+    int64_t numel;    /* elements = batch * tokens * hidden, > 0 */
+    int32_t group;    /* residual group in [0, n_groups) or -1 */
+    int32_t reserved; /* must be 0 */
+} cb_tensor_desc;
+
+enum {
+    CB_OK = 0,
+    CB_ERR_ARG = -1,               /* null, out-of-range or inconsistent argument */
+    CB_ERR_ALIGN = -2,             /* pointer not aligned to its element size (cache: 256 B) */
+    CB_ERR_NODES_DEGENERATE = -3,  /* duplicate node times: omega'(tau_j) = 0 (App. A) */
+    CB_ERR_HISTORY_NOT_FULL = -4,  /* fewer than K entries in H (Sec. 3.3 requires |H| = n) */
+    CB_ERR_ORDER = -5,             /* pushed time does not continue the sampling direction */
+    CB_ERR_UNBOUND = -6,           /* no cache arena bound to the plan */
+    CB_ERR_CUDA = -7,              /* a CUDA call or launch failed */
+    CB_ERR_LIMIT = -8              /* a size beyond CB_MAX_K / CB_MAX_TENSORS / CB_MAX_BRANCHES */
+};
+
+/* Full-computation schedule (Sec. 3.3, Eq. for F; Alg. 1 offline stage):
+ *   s in F  iff  s not in [s0, T-1-s1]  or  r divides (s - s0),   s in [0, T-1],
+ * then, when K > 0, every step whose history would hold fewer than K entries
+ * is also marked full (the text's "provided H contains enough entries").
+ * is_full: host array of T bytes, written 1 (full) or 0 (extrapolated).
+ * n_full: host int, receives the number of full steps (may be NULL).
+ * Errors: CB_ERR_ARG for T <= 0, r <= 0, s0 < 0, s1 < 0, K < 0 or is_full NULL. */
+int cb_schedule_full(int T, int r, int s0, int s1, int K, uint8_t* is_full, int* n_full);
+
+/* Offline precomputation (Sec. 3.3 "Weight Precomputation"; Alg. 1, offline
+ * stage). node_t: host array of the n_nodes timesteps at which full
+ * computations happen, in sampling order (strictly monotone). For every
+ * window of K consecutive nodes the fp64 barycentric weights rho_j of
+ * App. A, Eq. general_weights, are computed here on the normalised times
+ * tau = 2 (t - t_min) / (t_max - t_min) - 1. tensors: host array of n_tensors
+ * descriptors (copied). cache_dtype: storage type of the history buffer.
+ * out: receives the new plan. Errors: CB_ERR_ARG (K < 1, n_nodes < K, bad
+ * descriptor, t_min >= t_max, non-monotone nodes), CB_ERR_LIMIT,
+ * CB_ERR_NODES_DEGENERATE (repeated node time). */
+int cb_plan_create(const double* node_t, int n_nodes, int K, const cb_tensor_desc* tensors,
+                   int n_tensors, cb_dtype cache_dtype, double t_min, double t_max, cb_plan** out);
+
+/* Bytes of device memory the history buffer needs: K slots, each holding every
+ * tensor at a CB_CACHE_ALIGN-aligned offset. */
+size_t cb_plan_cache_bytes(const cb_plan* plan);
+
+/* Attach caller-owned device memory as the history buffer (the plan never
+ * allocates device memory). dev_ptr must be CB_CACHE_ALIGN-aligned and
+ * bytes >= cb_plan_cache_bytes. Rebinding empties the history.
+ * Errors: CB_ERR_ARG, CB_ERR_ALIGN. */
+int cb_plan_bind_cache(cb_plan* plan, void* dev_ptr, size_t bytes);
+
+/* Full step (Sec. 3.3; Alg. 1, full-computation branch): store the pair
+ * (t, f_t) in H. feats: host array of n_tensors device pointers, one per
+ * tensor descriptor, each numel elements of feat_dtype. One grouped kernel
+ * writes every tensor into the ring slot that holds the oldest entry (or the
+ * next free slot), converting fp32 -> bf16 (RNE) when the cache is bf16
+ * (bf16 -> bf16 is a bit copy, bf16 -> fp32 exact). t must continue the
+ * sampling direction of node_t strictly (CB_ERR_ORDER otherwise).
+ * Errors: CB_ERR_ARG, CB_ERR_ALIGN, CB_ERR_UNBOUND, CB_ERR_ORDER, CB_ERR_CUDA. */
+int cb_cache_push(cb_plan* plan, const void* const* feats, cb_dtype feat_dtype, double t, void* stream);
+
+/* Skipped step (Sec. 3.3, Eq. for f_t; Alg. 1, extrapolation branch): for
+ * every tensor i and element e,
+ *     P_i[e] = sum_j w_j(t_target) F_{i,j}[e]
+ * over the K entries of H, with the fp64 weights of Eq. barycentric_coeff
+ * computed on the host from the live node times. The weights travel as kernel
+ * parameters (an fp32 high/low pair each); one grouped persistent kernel
+ * covers all tensors, accumulating in fp32 with a compensated fallback, so
+ * that bf16 results are within one bf16 ulp of the exactly rounded value.
+ * outs: host array of n_tensors device pointers (entries may be NULL; the
+ *       array itself may be NULL), each receiving P_i as out_dtype.
+ * resid: host array of n_groups device pointers (may be NULL; entries may be
+ *       NULL). For group g, resid[g] <- round(resid[g] + sum_{i in g} P_i)
+ *       in place, with one rounding to resid_dtype (the block residual of
+ *       Sec. 3.1 with cached branches).
+ * A target equal to a node time returns that node's features exactly.
+ * Errors: CB_ERR_ARG, CB_ERR_ALIGN, CB_ERR_UNBOUND, CB_ERR_HISTORY_NOT_FULL,
+ * CB_ERR_CUDA. */
+int cb_extrapolate(cb_plan* plan, double t_target, void* const* outs, cb_dtype out_dtype,
+                   void* const* resid, cb_dtype resid_dtype, void* stream);
+
+/* As cb_extrapolate, for a history described by the caller (Sec. 3.3: H
+ * holds the n most recent pairs and the oldest is discarded, so a ring buffer
+ * holds them in rotated order). slot_t: host array of K times, slot_t[p]
+ * being the timestep whose features ring slot p holds; head: the slot of the
+ * OLDEST entry (logical order head, head+1, ... mod K). No data moves: only
+ * the weights are permuted to slot order. The plan's own history must be
+ * full (every slot written). Errors: as cb_extrapolate, plus
+ * CB_ERR_NODES_DEGENERATE for repeated slot times. */
+int cb_extrapolate_ring(cb_plan* plan, const double* slot_t, int head, double t_target,
+                        void* const* outs, cb_dtype out_dtype, void* const* resid,
+                        cb_dtype resid_dtype, void* stream);
+
+/* The fp64 weights cb_extrapolate would use for t_target on the live history
+ * (Eq. barycentric_coeff), in logical order oldest .. newest. w_logical: host
+ * array of K doubles. Errors: CB_ERR_ARG, CB_ERR_HISTORY_NOT_FULL. */
+int cb_weights(const cb_plan* plan, double t_target, double* w_logical);
+
+/* The "prepackaged" weight table (Sec. 3.3; Alg. 1, offline stage): for each
+ * targets[m] the weights over the K most recent nodes of node_t that precede
+ * it in sampling order, written to table[m*K + j] (j oldest .. newest).
+ * Errors: CB_ERR_ARG, CB_ERR_HISTORY_NOT_FULL (fewer than K nodes precede a
+ * target). */
+int cb_plan_export_weights(const cb_plan* plan, const double* targets, int n_targets, double* table);
+
+/* Introspection of H: slot_t (host, K doubles) receives each slot's time,
+ * head the slot of the oldest entry, count the number of entries (<= K).
+ * Any output pointer may be NULL. */
+int cb_plan_history(const cb_plan* plan, double* slot_t, int* head, int* count);
+
+/* Empty H (a new sample starts). */
+int cb_plan_reset(cb_plan* plan);
+
+/* Number of residual groups (1 + the largest descriptor group, 0 if none). */
+int cb_plan_num_groups(const cb_plan* plan);
+
+void cb_plan_destroy(cb_plan* plan);
+
+/* Static text for a status code. */
+const char* cb_status_string(int status);
+
+/* Text of the most recent CB_ERR_CUDA on the calling thread ("" if none). */
+const char* cb_last_error_message(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CHEBBOOST_H */

@@ -1,0 +1,193 @@
+"""ctypes binding of libchebboost (``include/chebboost.h``), same names, marshalling only.
+
+Every call forwards to the C ABI: pointers may be given as ints, ``None`` or any
+object with ``data_ptr()`` (a torch tensor); streams as ``None`` (legacy default
+stream), an int handle, or an object with ``cuda_stream`` (``torch.cuda.Stream``).
+A negative status raises :class:`CbError`. There is no fallback: importing this
+module fails if the compiled library is missing.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libchebboost.so")
+
+if not os.path.exists(LIB_PATH):
+    raise ImportError(
+        f"{LIB_PATH} is not built; run `python -m paper_2608_23429_gb300.build` "
+        "(the CUDA library is required, there is no CPU path)")
+
+_lib = ctypes.CDLL(LIB_PATH)
+
+CB_BF16, CB_FP32 = 0, 1
+CB_MAX_K, CB_MAX_TENSORS, CB_MAX_BRANCHES, CB_CACHE_ALIGN = 8, 256, 4, 256
+CB_OK, CB_ERR_ARG, CB_ERR_ALIGN, CB_ERR_NODES_DEGENERATE = 0, -1, -2, -3
+CB_ERR_HISTORY_NOT_FULL, CB_ERR_ORDER, CB_ERR_UNBOUND, CB_ERR_CUDA, CB_ERR_LIMIT = -4, -5, -6, -7, -8
+
+
+class cb_tensor_desc(ctypes.Structure):
+    _fields_ = [("layer", ctypes.c_int32), ("branch", ctypes.c_int32), ("numel", ctypes.c_int64),
+                ("group", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
+_P, _I, _D, _SZ = ctypes.c_void_p, ctypes.c_int, ctypes.c_double, ctypes.c_size_t
+_PP = ctypes.POINTER(ctypes.c_void_p)
+_sig = {
+    "cb_schedule_full": ([_I, _I, _I, _I, _I, _P, _P], _I),
+    "cb_plan_create": ([_P, _I, _I, _P, _I, _I, _D, _D, ctypes.POINTER(_P)], _I),
+    "cb_plan_cache_bytes": ([_P], _SZ),
+    "cb_plan_bind_cache": ([_P, _P, _SZ], _I),
+    "cb_cache_push": ([_P, _PP, _I, _D, _P], _I),
+    "cb_extrapolate": ([_P, _D, _PP, _I, _PP, _I, _P], _I),
+    "cb_extrapolate_ring": ([_P, _P, _I, _D, _PP, _I, _PP, _I, _P], _I),
+    "cb_weights": ([_P, _D, _P], _I),
+    "cb_plan_export_weights": ([_P, _P, _I, _P], _I),
+    "cb_plan_history": ([_P, _P, _P, _P], _I),
+    "cb_plan_reset": ([_P], _I),
+    "cb_plan_num_groups": ([_P], _I),
+    "cb_plan_destroy": ([_P], None),
+    "cb_status_string": ([_I], ctypes.c_char_p),
+    "cb_last_error_message": ([], ctypes.c_char_p),
+}
+for _name, (_args, _res) in _sig.items():
+    _f = getattr(_lib, _name)
+    _f.argtypes, _f.restype = _args, _res
+
+EXPORTED = tuple(_sig)
+
+
+class CbError(RuntimeError):
+    def __init__(self, status: int, call: str):
+        msg = _lib.cb_status_string(status).decode()
+        if status == CB_ERR_CUDA:
+            msg += ": " + _lib.cb_last_error_message().decode()
+        super().__init__(f"{call}: {msg} ({status})")
+        self.status = status
+
+
+def _check(rc: int, call: str) -> int:
+    if rc < 0:
+        raise CbError(rc, call)
+    return rc
+
+
+def _addr(x) -> int | None:
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    return int(x.data_ptr())
+
+
+def _ptr_array(xs):
+    if xs is None:
+        return None
+    return (ctypes.c_void_p * len(xs))(*[_addr(x) for x in xs])
+
+
+def _stream(s):
+    if s is None:
+        return None
+    if isinstance(s, int):
+        return s
+    return int(s.cuda_stream)
+
+
+def _f64(a):
+    return np.ascontiguousarray(a, dtype=np.float64)
+
+
+def cb_schedule_full(T: int, r: int, s0: int = 0, s1: int = 0, K: int = 0):
+    mask = np.zeros(T, dtype=np.uint8)
+    n = ctypes.c_int(0)
+    _check(_lib.cb_schedule_full(T, r, s0, s1, K, mask.ctypes.data, ctypes.byref(n)), "cb_schedule_full")
+    return mask.astype(bool), n.value
+
+
+def cb_plan_create(node_t, K: int, tensors, cache_dtype: int, t_min: float, t_max: float):
+    """``tensors``: sequence of (layer, branch, numel, group)."""
+    node_t = _f64(node_t)
+    descs = (cb_tensor_desc * len(tensors))(*[cb_tensor_desc(int(l), int(b), int(n), int(g), 0)
+                                             for (l, b, n, g) in tensors])
+    plan = ctypes.c_void_p()
+    _check(_lib.cb_plan_create(node_t.ctypes.data, node_t.size, K, ctypes.cast(descs, ctypes.c_void_p),
+                               len(tensors), cache_dtype, float(t_min), float(t_max), ctypes.byref(plan)),
+           "cb_plan_create")
+    return plan
+
+
+def cb_plan_cache_bytes(plan) -> int:
+    return int(_lib.cb_plan_cache_bytes(plan))
+
+
+def cb_plan_bind_cache(plan, dev_ptr, nbytes: int) -> None:
+    _check(_lib.cb_plan_bind_cache(plan, _addr(dev_ptr), nbytes), "cb_plan_bind_cache")
+
+
+def cb_cache_push(plan, feats, feat_dtype: int, t: float, stream=None) -> None:
+    _check(_lib.cb_cache_push(plan, _ptr_array(feats), feat_dtype, float(t), _stream(stream)), "cb_cache_push")
+
+
+def cb_extrapolate(plan, t_target: float, outs, out_dtype: int, resid=None, resid_dtype: int = CB_BF16,
+                   stream=None) -> None:
+    _check(_lib.cb_extrapolate(plan, float(t_target), _ptr_array(outs), out_dtype, _ptr_array(resid),
+                               resid_dtype, _stream(stream)), "cb_extrapolate")
+
+
+def cb_extrapolate_ring(plan, slot_t, head: int, t_target: float, outs, out_dtype: int, resid=None,
+                        resid_dtype: int = CB_BF16, stream=None) -> None:
+    slot_t = _f64(slot_t)
+    _check(_lib.cb_extrapolate_ring(plan, slot_t.ctypes.data, head, float(t_target), _ptr_array(outs),
+                                    out_dtype, _ptr_array(resid), resid_dtype, _stream(stream)),
+           "cb_extrapolate_ring")
+
+
+def cb_weights(plan, t_target: float, K: int) -> np.ndarray:
+    w = np.empty(K, dtype=np.float64)
+    _check(_lib.cb_weights(plan, float(t_target), w.ctypes.data), "cb_weights")
+    return w
+
+
+def cb_plan_export_weights(plan, targets, K: int) -> np.ndarray:
+    targets = _f64(targets)
+    table = np.empty((targets.size, K), dtype=np.float64)
+    _check(_lib.cb_plan_export_weights(plan, targets.ctypes.data, targets.size, table.ctypes.data),
+           "cb_plan_export_weights")
+    return table
+
+
+def cb_plan_history(plan, K: int):
+    slot_t = np.empty(K, dtype=np.float64)
+    head, count = ctypes.c_int(0), ctypes.c_int(0)
+    _check(_lib.cb_plan_history(plan, slot_t.ctypes.data, ctypes.byref(head), ctypes.byref(count)),
+           "cb_plan_history")
+    return slot_t, head.value, count.value
+
+
+def cb_plan_reset(plan) -> None:
+    _check(_lib.cb_plan_reset(plan), "cb_plan_reset")
+
+
+def cb_plan_num_groups(plan) -> int:
+    return int(_lib.cb_plan_num_groups(plan))
+
+
+def cb_plan_destroy(plan) -> None:
+    _lib.cb_plan_destroy(plan)
+
+
+def cb_status_string(status: int) -> str:
+    return _lib.cb_status_string(status).decode()
+
+
+def cb_last_error_message() -> str:
+    return _lib.cb_last_error_message().decode()
+
+
+def raw_status(name: str, *args) -> int:
+    """Call an entry point and return its status instead of raising (tests)."""
+    return getattr(_lib, name)(*args)

@@ -1,0 +1,68 @@
+// Internal: kernel argument blocks and launchers shared by the host plan
+// (plan.cpp) and the kernels (extrapolate.cu, push.cu). Not part of the ABI.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+namespace cbk {
+
+constexpr int kThreads = 256;     // threads per CTA
+constexpr int kVecElems = 8;      // elements per vector (16 B of bf16, 32 B of fp32)
+constexpr int kMaxItems = 256;    // work items (tensors, or residual groups) per launch
+constexpr int kMaxMembers = 256;  // branch tensors per launch
+
+// Vectors each thread handles per tile: two 16-B vectors for a bf16 cache,
+// one 32-B vector for an fp32 cache (both give 2*K 16-B loads in flight).
+__host__ __device__ constexpr int vectors_per_thread(bool cache_bf16) { return cache_bf16 ? 2 : 1; }
+__host__ __device__ constexpr long long tile_elems(bool cache_bf16) {
+    return (long long)kThreads * vectors_per_thread(cache_bf16) * kVecElems;
+}
+
+// One skipped-step launch. Items are the units of work: a single branch
+// tensor, or (with hidden states) all branch tensors of one residual group.
+// Every item is cut into tiles of tile_elems() elements; tiles are numbered
+// consecutively across items and dealt to a persistent grid.
+struct ExtrapArgs {
+    const unsigned char* cache;  // ring arena
+    long long slot_off[8];       // byte offset of history entry j (0 = oldest)
+    float w_hi[8];               // fp32(w_j)
+    float w_lo[8];               // fp32(w_j - w_hi[j])
+    float w_abs[8];              // |w_hi[j]| (error bound of the fast path)
+    int n_items;
+    int tiles_total;
+    int out_bf16;    // predictions are bf16 (else fp32)
+    int resid_bf16;  // hidden states are bf16 (else fp32)
+    int precise;     // 1: compensated (Dot2) arithmetic for every element
+    int tile_begin[kMaxItems + 1];
+    long long numel[kMaxItems];
+    void* resid[kMaxItems];           // hidden state of the item, or null
+    unsigned char nb[kMaxItems];      // member tensors of the item
+    unsigned char vec_ok[kMaxItems];  // every pointer of the item is 16-B aligned
+    short first[kMaxItems];           // first member index
+    long long m_off[kMaxMembers];     // byte offset of the member tensor inside one slot
+    void* m_out[kMaxMembers];         // prediction output of the member, or null
+};
+
+// One full-step launch: copy/convert every tensor into one ring slot.
+struct PushArgs {
+    unsigned char* slot;  // base of the destination slot
+    int n_items;
+    int tiles_total;
+    int tile_begin[kMaxItems + 1];
+    long long numel[kMaxItems];
+    long long off[kMaxItems];  // byte offset of the tensor inside the slot
+    const void* src[kMaxItems];
+    unsigned char vec_ok[kMaxItems];
+};
+
+constexpr long long push_tile_elems = (long long)kThreads * 2 * kVecElems;
+
+cudaError_t launch_extrapolate(const ExtrapArgs& a, int K, bool cache_bf16, int grid, cudaStream_t s);
+cudaError_t extrapolate_blocks_per_sm(int K, bool cache_bf16, int* blocks);
+
+cudaError_t launch_push(const PushArgs& a, bool src_bf16, bool dst_bf16, int grid, cudaStream_t s);
+cudaError_t push_blocks_per_sm(bool src_bf16, bool dst_bf16, int* blocks);
+
+}  // namespace cbk

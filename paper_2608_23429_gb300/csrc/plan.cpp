@@ -1,0 +1,516 @@
+// Host side of libchebboost: the plan (offline precomputation, Sec. 3.3
+// "Weight Precomputation"; Alg. 1 offline stage), the history buffer's ring
+// bookkeeping, the online weights (Sec. 3.2 Eq. barycentric_coeff) and the
+// launches of the two kernels. Everything here is fp64 host arithmetic that
+// runs in microseconds per call; all device work is in push.cu and
+// extrapolate.cu.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <memory>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "../../include/chebboost.h"
+#include "cb_device.h"
+
+namespace {
+
+thread_local std::string g_last_error;
+
+int cuda_fail(cudaError_t e, const char* where) {
+    g_last_error = std::string(where) + ": " + cudaGetErrorName(e) + ": " + cudaGetErrorString(e);
+    return CB_ERR_CUDA;
+}
+
+size_t esize(cb_dtype d) { return d == CB_BF16 ? 2 : 4; }
+bool valid_dtype(cb_dtype d) { return d == CB_BF16 || d == CB_FP32; }
+size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Barycentric weights rho_j = 1 / prod_{k != j} (x_j - x_k) (App. A, Eq. general_weights).
+bool rho_of(const double* x, int n, double* rho) {
+    for (int j = 0; j < n; ++j) {
+        double d = 1.0;
+        for (int k = 0; k < n; ++k)
+            if (k != j) d *= x[j] - x[k];
+        if (d == 0.0 || !std::isfinite(d)) return false;
+        rho[j] = 1.0 / d;
+    }
+    return true;
+}
+
+// Interpolation coefficients w_j = (rho_j / (x - x_j)) / sum_i rho_i / (x - x_i)
+// (Sec. 3.2, Eq. barycentric_coeff). A target on a node gives the unit vector.
+void coeff_of(const double* x, const double* rho, int n, double xq, double* w) {
+    for (int j = 0; j < n; ++j)
+        if (xq == x[j]) {
+            for (int i = 0; i < n; ++i) w[i] = (i == j) ? 1.0 : 0.0;
+            return;
+        }
+    double den = 0.0;
+    for (int i = 0; i < n; ++i) {
+        w[i] = rho[i] / (xq - x[i]);
+        den += w[i];
+    }
+    for (int i = 0; i < n; ++i) w[i] /= den;
+}
+
+struct DeviceInfo {
+    int device = -1;
+    int sms = 0;
+    int occ_extrap[2][CB_MAX_K + 1] = {};  // [cache_bf16][K]
+    int occ_push[2][2] = {};               // [src_bf16][dst_bf16]
+};
+
+}  // namespace
+
+struct cb_plan {
+    int K = 0;
+    cb_dtype cache_dtype = CB_BF16;
+    double t_min = 0, t_max = 1;
+    std::vector<cb_tensor_desc> tensors;
+    std::vector<std::vector<int>> groups;  // residual group -> member tensors
+    std::vector<double> node_t;            // full-step timesteps, sampling order
+    std::vector<double> node_tau;
+    int dir = 0;                           // +1 increasing, -1 decreasing t
+    std::vector<double> rho_win;           // rho of node window i: rho_win[i*K + j]
+    std::vector<long long> off;            // byte offset of tensor i inside a slot
+    size_t slot_bytes = 0;
+    // bound history buffer
+    unsigned char* cache = nullptr;
+    // ring state of H
+    double slot_t[CB_MAX_K] = {};
+    int next = 0;   // slot written by the next push
+    int count = 0;  // entries held (<= K)
+    bool has_last = false;
+    double last_t = 0;
+    DeviceInfo dev;
+    std::unique_ptr<cbk::ExtrapArgs> eargs{new cbk::ExtrapArgs};
+    std::unique_ptr<cbk::PushArgs> pargs{new cbk::PushArgs};
+
+    double tau(double t) const { return 2.0 * (t - t_min) / (t_max - t_min) - 1.0; }
+    int oldest() const { return count < K ? 0 : next; }
+};
+
+namespace {
+
+int ensure_device(cb_plan* p) {
+    int d = 0;
+    cudaError_t e = cudaGetDevice(&d);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (p->dev.device != d) {
+        DeviceInfo info;
+        info.device = d;
+        e = cudaDeviceGetAttribute(&info.sms, cudaDevAttrMultiProcessorCount, d);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
+        p->dev = info;
+    }
+    return CB_OK;
+}
+
+int extrap_grid(cb_plan* p, int K, bool cb16, int tiles, int* grid) {
+    int& occ = p->dev.occ_extrap[cb16 ? 1 : 0][K];
+    if (occ == 0) {
+        cudaError_t e = cbk::extrapolate_blocks_per_sm(K, cb16, &occ);
+        if (e != cudaSuccess || occ <= 0) {
+            occ = 0;
+            return cuda_fail(e == cudaSuccess ? cudaErrorInvalidConfiguration : e, "occupancy");
+        }
+    }
+    long long g = (long long)p->dev.sms * occ;
+    *grid = (int)(tiles < g ? tiles : g);
+    return CB_OK;
+}
+
+int push_grid(cb_plan* p, bool sb, bool db, int tiles, int* grid) {
+    int& occ = p->dev.occ_push[sb ? 1 : 0][db ? 1 : 0];
+    if (occ == 0) {
+        cudaError_t e = cbk::push_blocks_per_sm(sb, db, &occ);
+        if (e != cudaSuccess || occ <= 0) {
+            occ = 0;
+            return cuda_fail(e == cudaSuccess ? cudaErrorInvalidConfiguration : e, "occupancy");
+        }
+    }
+    long long g = (long long)p->dev.sms * occ;
+    *grid = (int)(tiles < g ? tiles : g);
+    return CB_OK;
+}
+
+bool aligned(const void* ptr, size_t a) { return ((uintptr_t)ptr % a) == 0; }
+
+// Logical history times (oldest first) and the slot of each entry.
+struct Window {
+    double t[CB_MAX_K];
+    double tau[CB_MAX_K];
+    int slot[CB_MAX_K];
+};
+
+// rho for a window: reuse the offline table when the window is K consecutive
+// nodes of the plan, otherwise compute it the same way now.
+bool window_rho(const cb_plan* p, const Window& w, double* rho) {
+    const int K = p->K;
+    const int n = (int)p->node_t.size();
+    for (int i = 0; i + K <= n; ++i) {
+        if (p->node_t[i] != w.t[0]) continue;
+        bool match = true;
+        for (int j = 1; j < K && match; ++j) match = p->node_t[i + j] == w.t[j];
+        if (match) {
+            std::memcpy(rho, &p->rho_win[(size_t)i * K], sizeof(double) * K);
+            return true;
+        }
+    }
+    return rho_of(w.tau, K, rho);
+}
+
+int weights_for(const cb_plan* p, const Window& w, double t_target, double* out) {
+    if (!std::isfinite(t_target)) return CB_ERR_ARG;
+    double rho[CB_MAX_K];
+    if (!window_rho(p, w, rho)) return CB_ERR_NODES_DEGENERATE;
+    for (int j = 0; j < p->K; ++j)
+        if (t_target == w.t[j]) {  // the target is a cached node: return it exactly
+            for (int i = 0; i < p->K; ++i) out[i] = (i == j) ? 1.0 : 0.0;
+            return CB_OK;
+        }
+    coeff_of(w.tau, rho, p->K, p->tau(t_target), out);
+    return CB_OK;
+}
+
+Window live_window(const cb_plan* p) {
+    Window w{};
+    const int o = p->oldest();
+    for (int j = 0; j < p->K; ++j) {
+        w.slot[j] = (o + j) % p->K;
+        w.t[j] = p->slot_t[w.slot[j]];
+        w.tau[j] = p->tau(w.t[j]);
+    }
+    return w;
+}
+
+int run_extrapolate(cb_plan* p, const Window& win, double t_target, void* const* outs, cb_dtype out_dtype,
+                    void* const* resid, cb_dtype resid_dtype, void* stream) {
+    if (!p->cache) return CB_ERR_UNBOUND;
+    if (p->count < p->K) return CB_ERR_HISTORY_NOT_FULL;
+    if (!valid_dtype(out_dtype) || !valid_dtype(resid_dtype)) return CB_ERR_ARG;
+    const int n = (int)p->tensors.size();
+    const int ng = (int)p->groups.size();
+    const size_t oes = esize(out_dtype), res = esize(resid_dtype);
+    if (outs)
+        for (int i = 0; i < n; ++i)
+            if (outs[i] && !aligned(outs[i], oes)) return CB_ERR_ALIGN;
+    if (resid)
+        for (int g = 0; g < ng; ++g)
+            if (resid[g] && !aligned(resid[g], res)) return CB_ERR_ALIGN;
+
+    double w[CB_MAX_K];
+    int rc = weights_for(p, win, t_target, w);
+    if (rc != CB_OK) return rc;
+
+    cbk::ExtrapArgs& A = *p->eargs;
+    const bool cb16 = p->cache_dtype == CB_BF16;
+    const long long te = cbk::tile_elems(cb16);
+    A.cache = p->cache;
+    for (int j = 0; j < CB_MAX_K; ++j) {
+        const bool on = j < p->K;
+        A.slot_off[j] = on ? (long long)win.slot[j] * (long long)p->slot_bytes : 0;
+        const float hi = on ? (float)w[j] : 0.0f;
+        A.w_hi[j] = hi;
+        A.w_lo[j] = on ? (float)(w[j] - (double)hi) : 0.0f;
+        A.w_abs[j] = std::fabs(hi);
+    }
+    A.out_bf16 = out_dtype == CB_BF16;
+    A.resid_bf16 = resid_dtype == CB_BF16;
+
+    int items = 0, members = 0;
+    long long tiles = 0;
+    bool any_out = false, any_resid = false;
+    auto add_item = [&](const int* mem, int nm, void* res_ptr) {
+        const long long numel = p->tensors[mem[0]].numel;
+        bool vec = !res_ptr || aligned(res_ptr, 16);
+        A.first[items] = (short)members;
+        for (int m = 0; m < nm; ++m) {
+            const int i = mem[m];
+            void* o = outs ? outs[i] : nullptr;
+            A.m_off[members] = p->off[i];
+            A.m_out[members] = o;
+            if (o) {
+                any_out = true;
+                vec = vec && aligned(o, 16);
+            }
+            ++members;
+        }
+        if (res_ptr) any_resid = true;
+        A.nb[items] = (unsigned char)nm;
+        A.resid[items] = res_ptr;
+        A.vec_ok[items] = vec ? 1 : 0;
+        A.numel[items] = numel;
+        A.tile_begin[items] = (int)tiles;
+        tiles += (numel + te - 1) / te;
+        ++items;
+    };
+    std::vector<char> grouped(n, 0);
+    if (resid)
+        for (int g = 0; g < ng; ++g)
+            if (resid[g] && !p->groups[g].empty()) {
+                add_item(p->groups[g].data(), (int)p->groups[g].size(), resid[g]);
+                for (int i : p->groups[g]) grouped[i] = 1;
+            }
+    for (int i = 0; i < n; ++i)
+        if (!grouped[i] && outs && outs[i]) add_item(&i, 1, nullptr);
+    if (tiles > 0x7FFFFFFFLL) return CB_ERR_LIMIT;
+    A.tile_begin[items] = (int)tiles;
+    A.n_items = items;
+    A.tiles_total = (int)tiles;
+    A.precise = (any_out && out_dtype == CB_FP32) || (any_resid && resid_dtype == CB_FP32);
+    if (items == 0) return CB_OK;  // nothing requested
+
+    rc = ensure_device(p);
+    if (rc != CB_OK) return rc;
+    int grid = 0;
+    rc = extrap_grid(p, p->K, cb16, (int)tiles, &grid);
+    if (rc != CB_OK) return rc;
+    cudaError_t e = cbk::launch_extrapolate(A, p->K, cb16, grid, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, "extrapolate launch");
+    return CB_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int cb_schedule_full(int T, int r, int s0, int s1, int K, uint8_t* is_full, int* n_full) {
+    if (T <= 0 || r <= 0 || s0 < 0 || s1 < 0 || K < 0 || !is_full) return CB_ERR_ARG;
+    int held = 0, nf = 0;
+    for (int s = 0; s < T; ++s) {
+        const bool in_range = s >= s0 && s <= T - 1 - s1;
+        bool full = !in_range || (s - s0) % r == 0;
+        if (held < K) full = true;  // not enough history to extrapolate yet
+        is_full[s] = full ? 1 : 0;
+        if (full) {
+            ++nf;
+            if (held < K) ++held;
+        }
+    }
+    if (n_full) *n_full = nf;
+    return CB_OK;
+}
+
+int cb_plan_create(const double* node_t, int n_nodes, int K, const cb_tensor_desc* tensors, int n_tensors,
+                   cb_dtype cache_dtype, double t_min, double t_max, cb_plan** out) {
+    if (!out) return CB_ERR_ARG;
+    *out = nullptr;
+    if (K < 1 || K > CB_MAX_K) return K < 1 ? CB_ERR_ARG : CB_ERR_LIMIT;
+    if (!node_t || n_nodes < K || !tensors || n_tensors < 1) return CB_ERR_ARG;
+    if (n_tensors > CB_MAX_TENSORS) return CB_ERR_LIMIT;
+    if (!valid_dtype(cache_dtype)) return CB_ERR_ARG;
+    if (!(std::isfinite(t_min) && std::isfinite(t_max) && t_min < t_max)) return CB_ERR_ARG;
+    for (int i = 0; i < n_nodes; ++i)
+        if (!std::isfinite(node_t[i])) return CB_ERR_ARG;
+    int dir = 0;
+    if (n_nodes >= 2) {
+        for (int i = 1; i < n_nodes; ++i) {
+            const double d = node_t[i] - node_t[i - 1];
+            if (d == 0.0) return CB_ERR_NODES_DEGENERATE;
+            const int s = d > 0 ? 1 : -1;
+            if (dir == 0) dir = s;
+            if (s != dir) return CB_ERR_ARG;  // nodes must be strictly monotone
+        }
+    }
+    try {
+        std::unique_ptr<cb_plan> p(new cb_plan);
+        p->K = K;
+        p->cache_dtype = cache_dtype;
+        p->t_min = t_min;
+        p->t_max = t_max;
+        p->dir = dir;
+        p->tensors.assign(tensors, tensors + n_tensors);
+        int ng = 0;
+        for (const auto& d : p->tensors) {
+            if (d.numel <= 0 || d.reserved != 0 || d.group < -1) return CB_ERR_ARG;
+            if (d.group + 1 > ng) ng = d.group + 1;
+        }
+        if (ng > cbk::kMaxItems) return CB_ERR_LIMIT;
+        p->groups.assign(ng, {});
+        for (int i = 0; i < n_tensors; ++i) {
+            const auto& d = p->tensors[i];
+            if (d.group < 0) continue;
+            auto& g = p->groups[d.group];
+            if (!g.empty() && p->tensors[g[0]].numel != d.numel) return CB_ERR_ARG;
+            g.push_back(i);
+            if ((int)g.size() > CB_MAX_BRANCHES) return CB_ERR_LIMIT;
+        }
+        p->node_t.assign(node_t, node_t + n_nodes);
+        p->node_tau.resize(n_nodes);
+        for (int i = 0; i < n_nodes; ++i) p->node_tau[i] = p->tau(node_t[i]);
+        // offline stage: rho for every window of K consecutive nodes
+        p->rho_win.resize((size_t)(n_nodes - K + 1) * K);
+        for (int i = 0; i + K <= n_nodes; ++i)
+            if (!rho_of(&p->node_tau[i], K, &p->rho_win[(size_t)i * K])) return CB_ERR_NODES_DEGENERATE;
+        // slot layout: tensors back to back, each at a CB_CACHE_ALIGN boundary
+        size_t o = 0;
+        p->off.resize(n_tensors);
+        for (int i = 0; i < n_tensors; ++i) {
+            p->off[i] = (long long)o;
+            o = round_up(o + (size_t)p->tensors[i].numel * esize(cache_dtype), CB_CACHE_ALIGN);
+        }
+        p->slot_bytes = o;
+        *out = p.release();
+        return CB_OK;
+    } catch (const std::bad_alloc&) {
+        return CB_ERR_LIMIT;
+    }
+}
+
+size_t cb_plan_cache_bytes(const cb_plan* p) { return p ? p->slot_bytes * (size_t)p->K : 0; }
+
+int cb_plan_bind_cache(cb_plan* p, void* dev_ptr, size_t bytes) {
+    if (!p || !dev_ptr || bytes < cb_plan_cache_bytes(p)) return CB_ERR_ARG;
+    if (!aligned(dev_ptr, CB_CACHE_ALIGN)) return CB_ERR_ALIGN;
+    p->cache = static_cast<unsigned char*>(dev_ptr);
+    p->next = p->count = 0;
+    p->has_last = false;
+    return CB_OK;
+}
+
+int cb_cache_push(cb_plan* p, const void* const* feats, cb_dtype feat_dtype, double t, void* stream) {
+    if (!p || !feats || !valid_dtype(feat_dtype) || !std::isfinite(t)) return CB_ERR_ARG;
+    if (!p->cache) return CB_ERR_UNBOUND;
+    const int n = (int)p->tensors.size();
+    const size_t fes = esize(feat_dtype);
+    for (int i = 0; i < n; ++i) {
+        if (!feats[i]) return CB_ERR_ARG;
+        if (!aligned(feats[i], fes)) return CB_ERR_ALIGN;
+    }
+    if (p->has_last) {
+        const double d = t - p->last_t;
+        if (d == 0.0 || (p->dir != 0 && (d > 0 ? 1 : -1) != p->dir)) return CB_ERR_ORDER;
+    }
+    for (int j = 0; j < p->count; ++j)
+        if (p->slot_t[(p->oldest() + j) % p->K] == t) return CB_ERR_NODES_DEGENERATE;
+
+    cbk::PushArgs& A = *p->pargs;
+    const bool sb = feat_dtype == CB_BF16, db = p->cache_dtype == CB_BF16;
+    A.slot = p->cache + (size_t)p->next * p->slot_bytes;
+    long long tiles = 0;
+    for (int i = 0; i < n; ++i) {
+        A.tile_begin[i] = (int)tiles;
+        A.numel[i] = p->tensors[i].numel;
+        A.off[i] = p->off[i];
+        A.src[i] = feats[i];
+        A.vec_ok[i] = aligned(feats[i], 16) ? 1 : 0;
+        tiles += (p->tensors[i].numel + cbk::push_tile_elems - 1) / cbk::push_tile_elems;
+    }
+    if (tiles > 0x7FFFFFFFLL) return CB_ERR_LIMIT;
+    A.tile_begin[n] = (int)tiles;
+    A.n_items = n;
+    A.tiles_total = (int)tiles;
+    int rc = ensure_device(p);
+    if (rc != CB_OK) return rc;
+    int grid = 0;
+    rc = push_grid(p, sb, db, (int)tiles, &grid);
+    if (rc != CB_OK) return rc;
+    cudaError_t e = cbk::launch_push(A, sb, db, grid, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, "push launch");
+    // the pair (t, f_t) is now in H; the oldest entry was overwritten when full
+    p->slot_t[p->next] = t;
+    p->next = (p->next + 1) % p->K;
+    if (p->count < p->K) ++p->count;
+    p->has_last = true;
+    p->last_t = t;
+    return CB_OK;
+}
+
+int cb_extrapolate(cb_plan* p, double t_target, void* const* outs, cb_dtype out_dtype, void* const* resid,
+                   cb_dtype resid_dtype, void* stream) {
+    if (!p) return CB_ERR_ARG;
+    if (p->count < p->K) return p->cache ? CB_ERR_HISTORY_NOT_FULL : CB_ERR_UNBOUND;
+    return run_extrapolate(p, live_window(p), t_target, outs, out_dtype, resid, resid_dtype, stream);
+}
+
+int cb_extrapolate_ring(cb_plan* p, const double* slot_t, int head, double t_target, void* const* outs,
+                        cb_dtype out_dtype, void* const* resid, cb_dtype resid_dtype, void* stream) {
+    if (!p || !slot_t || head < 0 || head >= (p ? p->K : 1)) return CB_ERR_ARG;
+    if (p->count < p->K) return p->cache ? CB_ERR_HISTORY_NOT_FULL : CB_ERR_UNBOUND;
+    Window w{};
+    for (int j = 0; j < p->K; ++j) {
+        w.slot[j] = (head + j) % p->K;
+        w.t[j] = slot_t[w.slot[j]];
+        if (!std::isfinite(w.t[j])) return CB_ERR_ARG;
+        w.tau[j] = p->tau(w.t[j]);
+        for (int i = 0; i < j; ++i)
+            if (w.t[i] == w.t[j]) return CB_ERR_NODES_DEGENERATE;
+    }
+    return run_extrapolate(p, w, t_target, outs, out_dtype, resid, resid_dtype, stream);
+}
+
+int cb_weights(const cb_plan* p, double t_target, double* w_logical) {
+    if (!p || !w_logical) return CB_ERR_ARG;
+    if (p->count < p->K) return CB_ERR_HISTORY_NOT_FULL;
+    return weights_for(p, live_window(p), t_target, w_logical);
+}
+
+int cb_plan_export_weights(const cb_plan* p, const double* targets, int n_targets, double* table) {
+    if (!p || (n_targets > 0 && (!targets || !table)) || n_targets < 0) return CB_ERR_ARG;
+    const int K = p->K, n = (int)p->node_t.size();
+    for (int m = 0; m < n_targets; ++m) {
+        const double t = targets[m];
+        if (!std::isfinite(t)) return CB_ERR_ARG;
+        // the K most recent nodes that precede t in sampling order
+        int last = -1;
+        for (int i = 0; i < n; ++i) {
+            const double d = t - p->node_t[i];
+            const bool before = p->dir >= 0 ? d > 0 : d < 0;
+            if (before) last = i;
+        }
+        if (last + 1 < K) return CB_ERR_HISTORY_NOT_FULL;
+        Window w{};
+        for (int j = 0; j < K; ++j) {
+            w.t[j] = p->node_t[last - K + 1 + j];
+            w.tau[j] = p->node_tau[last - K + 1 + j];
+        }
+        const int rc = weights_for(p, w, t, &table[(size_t)m * K]);
+        if (rc != CB_OK) return rc;
+    }
+    return CB_OK;
+}
+
+int cb_plan_history(const cb_plan* p, double* slot_t, int* head, int* count) {
+    if (!p) return CB_ERR_ARG;
+    if (slot_t)
+        for (int j = 0; j < p->K; ++j) slot_t[j] = p->slot_t[j];
+    if (head) *head = p->oldest();
+    if (count) *count = p->count;
+    return CB_OK;
+}
+
+int cb_plan_reset(cb_plan* p) {
+    if (!p) return CB_ERR_ARG;
+    p->next = p->count = 0;
+    p->has_last = false;
+    return CB_OK;
+}
+
+int cb_plan_num_groups(const cb_plan* p) { return p ? (int)p->groups.size() : 0; }
+
+void cb_plan_destroy(cb_plan* p) { delete p; }
+
+const char* cb_status_string(int s) {
+    switch (s) {
+    case CB_OK: return "ok";
+    case CB_ERR_ARG: return "invalid argument";
+    case CB_ERR_ALIGN: return "misaligned pointer";
+    case CB_ERR_NODES_DEGENERATE: return "duplicate node times (omega'(tau_j) = 0)";
+    case CB_ERR_HISTORY_NOT_FULL: return "history buffer holds fewer than K entries";
+    case CB_ERR_ORDER: return "pushed time does not continue the sampling direction";
+    case CB_ERR_UNBOUND: return "no cache arena bound to the plan";
+    case CB_ERR_CUDA: return "CUDA error";
+    case CB_ERR_LIMIT: return "size limit exceeded";
+    default: return "unknown status";
+    }
+}
+
+const char* cb_last_error_message(void) { return g_last_error.c_str(); }
+
+}  // extern "C"

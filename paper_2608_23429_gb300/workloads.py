@@ -171,14 +171,21 @@ def _tau(w: Workload, t: float) -> float:
     return 2.0 * (t - w.t_min) / (w.t_max - w.t_min) - 1.0
 
 
-def trajectory(w: Workload, i: int, t: float, node_index: int, device, out_dtype=None) -> torch.Tensor:
-    """Branch output ``i`` at timestep ``t`` (the value a full step would cache)."""
+def trajectory(w: Workload, i: int, t: float, node_index: int, device, out_dtype=None,
+               exact: bool = False, absolute: bool = False) -> torch.Tensor:
+    """Branch output ``i`` at timestep ``t`` (the value a full step would cache).
+
+    With ``exact`` the noise-free series is summed in fp64 from the same fp32
+    coefficients (the analytic trajectory); with ``absolute`` as well, each
+    term enters with its magnitude (a bound on the rounding of the fp32 sum).
+    """
     spec = w.tensors[i]
     dev = torch.device(device)
     g = torch.Generator(device=dev)
     g.manual_seed(_seed(w.seed, i, 1))
     tau = _tau(w, t)
-    F = torch.zeros(spec.shape, dtype=torch.float32, device=dev)
+    acc_dt = torch.float64 if exact else torch.float32
+    F = torch.zeros(spec.shape, dtype=acc_dt, device=dev)
     t_prev, t_cur = 1.0, tau  # T_0, T_1
     for d in range(w.degree + 1):
         c = torch.randn(spec.shape, generator=g, device=dev, dtype=torch.float32)
@@ -186,15 +193,23 @@ def trajectory(w: Workload, i: int, t: float, node_index: int, device, out_dtype
         if d >= 2:
             t_prev, t_cur = t_cur, 2.0 * tau * t_cur - t_prev
             Td = t_cur
-        F.add_(c, alpha=Td / float((d + 1) ** 2))
+        if absolute:
+            F.add_(c.to(acc_dt).abs(), alpha=abs(Td) / float((d + 1) ** 2))
+        else:
+            F.add_(c.to(acc_dt), alpha=Td / float((d + 1) ** 2))
+    if w.lognormal:
+        gs = torch.Generator(device=dev)
+        gs.manual_seed(_seed(w.seed, i, 3))
+        scale = torch.exp(torch.randn(spec.shape[-1], generator=gs, device=dev, dtype=torch.float32))
+    if exact:
+        if w.lognormal:
+            F.mul_(scale.to(acc_dt))
+        return F if out_dtype is None else F.to(out_dtype)
     if w.noise > 0:
         gn = torch.Generator(device=dev)
         gn.manual_seed(_seed(w.seed, i, 2, node_index))
         F.add_(torch.randn(spec.shape, generator=gn, device=dev, dtype=torch.float32), alpha=w.noise)
     if w.lognormal:
-        gs = torch.Generator(device=dev)
-        gs.manual_seed(_seed(w.seed, i, 3))
-        scale = torch.exp(torch.randn(spec.shape[-1], generator=gs, device=dev, dtype=torch.float32))
         F.mul_(scale)
     dt = out_dtype or (torch.bfloat16 if w.cache_dtype == "bf16" else torch.float32)
     return F.to(dt)

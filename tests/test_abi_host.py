@@ -1,0 +1,179 @@
+"""C ABI and host logic of libchebboost, on the CPU.
+
+No test here launches a kernel: they cover the exported symbols, the
+host-side schedule and weight precomputation (against the oracle), the slot
+layout and every validation error that is returned before a launch.
+"""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def cb():
+    from paper_2608_23429_gb300 import build
+    build.build()
+    from paper_2608_23429_gb300 import chebboost
+    return chebboost
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "chebboost.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(cb_\w+)\s*\(", src)))
+
+
+def test_every_declared_symbol_is_exported(cb):
+    names = _declared()
+    assert len(names) >= 15
+    lib = ctypes.CDLL(cb.LIB_PATH)
+    for n in names:
+        assert hasattr(lib, n), n
+    assert set(names) <= set(cb.EXPORTED)
+
+
+def test_status_strings(cb):
+    for s in range(0, -9, -1):
+        assert cb.cb_status_string(s) and cb.cb_status_string(s) != "unknown status"
+
+
+def test_schedule_matches_oracle(cb, orc):
+    rng = np.random.default_rng(3)
+    for _ in range(300):
+        T = int(rng.integers(1, 60))
+        r = int(rng.integers(1, 9))
+        s0, s1, K = int(rng.integers(0, 6)), int(rng.integers(0, 6)), int(rng.integers(0, 9))
+        mask, n = cb.cb_schedule_full(T, r, s0, s1, K)
+        ref = orc.full_schedule(T, r, s0, s1, K)
+        assert np.array_equal(mask, ref), (T, r, s0, s1, K)
+        assert n == int(ref.sum())
+
+
+def _tensors(numels, groups=None):
+    groups = groups or [-1] * len(numels)
+    return [(i, 0, n, g) for i, (n, g) in enumerate(zip(numels, groups))]
+
+
+def test_plan_create_errors(cb):
+    E = cb.CbError
+    nodes = [999.0, 900.0, 800.0, 700.0]
+    ok = _tensors([100, 100])
+
+    def status(**kw):
+        args = dict(node_t=nodes, K=3, tensors=ok, cache_dtype=cb.CB_BF16, t_min=0.0, t_max=999.0)
+        args.update(kw)
+        try:
+            p = cb.cb_plan_create(**args)
+        except E as e:
+            return e.status
+        cb.cb_plan_destroy(p)
+        return 0
+
+    assert status() == 0
+    assert status(K=0) == cb.CB_ERR_ARG
+    assert status(K=9) == cb.CB_ERR_LIMIT
+    assert status(node_t=nodes[:2]) == cb.CB_ERR_ARG
+    assert status(node_t=[999.0, 900.0, 900.0, 700.0]) == cb.CB_ERR_NODES_DEGENERATE
+    assert status(node_t=[999.0, 900.0, 950.0, 700.0]) == cb.CB_ERR_ARG
+    assert status(t_min=5.0, t_max=5.0) == cb.CB_ERR_ARG
+    assert status(t_min=float("nan")) == cb.CB_ERR_ARG
+    assert status(cache_dtype=7) == cb.CB_ERR_ARG
+    assert status(tensors=_tensors([100, 0])) == cb.CB_ERR_ARG
+    assert status(tensors=_tensors([100, 101], [0, 0])) == cb.CB_ERR_ARG  # group numel mismatch
+    assert status(tensors=_tensors([8] * 5, [0] * 5)) == cb.CB_ERR_LIMIT  # > CB_MAX_BRANCHES
+    assert status(tensors=_tensors([8] * 257)) == cb.CB_ERR_LIMIT
+    assert status(tensors=[(0, 0, 8, -2)]) == cb.CB_ERR_ARG
+
+
+def test_cache_layout_and_bind(cb):
+    numels = [1, 7, 128, 129, 1000]
+    for dt, es in ((cb.CB_BF16, 2), (cb.CB_FP32, 4)):
+        p = cb.cb_plan_create([3.0, 2.0, 1.0], 3, _tensors(numels), dt, 0.0, 3.0)
+        slot = sum((n * es + 255) // 256 * 256 for n in numels)
+        assert cb.cb_plan_cache_bytes(p) == 3 * slot
+        with pytest.raises(cb.CbError) as e:
+            cb.cb_plan_bind_cache(p, 0x1000 + 128, 3 * slot)
+        assert e.value.status == cb.CB_ERR_ALIGN
+        with pytest.raises(cb.CbError) as e:
+            cb.cb_plan_bind_cache(p, 0x1000, 3 * slot - 1)
+        assert e.value.status == cb.CB_ERR_ARG
+        cb.cb_plan_destroy(p)
+
+
+def test_validation_before_launch(cb):
+    """Every error below is returned before any CUDA call (safe with or without a GPU)."""
+    p = cb.cb_plan_create([999.0, 900.0, 800.0], 3, _tensors([64, 64], [0, 0]), cb.CB_BF16, 0.0, 999.0)
+    st = cb.raw_status
+    arr = lambda *xs: (ctypes.c_void_p * len(xs))(*xs)
+    # unbound
+    assert st("cb_cache_push", p, arr(0x1000, 0x2000), 0, 999.0, None) == cb.CB_ERR_UNBOUND
+    assert st("cb_extrapolate", p, 850.0, arr(0x1000, 0x2000), 0, None, 0, None) == cb.CB_ERR_UNBOUND
+    cb.cb_plan_bind_cache(p, 0x100000, cb.cb_plan_cache_bytes(p))  # never dereferenced below
+    assert st("cb_cache_push", p, None, 0, 999.0, None) == cb.CB_ERR_ARG
+    assert st("cb_cache_push", p, arr(0x1000, 0), 0, 999.0, None) == cb.CB_ERR_ARG
+    assert st("cb_cache_push", p, arr(0x1001, 0x2000), 0, 999.0, None) == cb.CB_ERR_ALIGN
+    assert st("cb_cache_push", p, arr(0x1002, 0x2000), 1, 999.0, None) == cb.CB_ERR_ALIGN
+    assert st("cb_cache_push", p, arr(0x1000, 0x2000), 5, 999.0, None) == cb.CB_ERR_ARG
+    assert st("cb_cache_push", p, arr(0x1000, 0x2000), 0, float("inf"), None) == cb.CB_ERR_ARG
+    # history not full
+    assert st("cb_extrapolate", p, 850.0, arr(0x1000, 0x2000), 0, None, 0, None) == cb.CB_ERR_HISTORY_NOT_FULL
+    assert st("cb_extrapolate_ring", p, (ctypes.c_double * 3)(1, 2, 3), 0, 850.0, None, 0, None, 0,
+              None) == cb.CB_ERR_HISTORY_NOT_FULL
+    assert st("cb_extrapolate_ring", p, (ctypes.c_double * 3)(1, 2, 3), 3, 850.0, None, 0, None, 0,
+              None) == cb.CB_ERR_ARG
+    w = (ctypes.c_double * 3)()
+    assert st("cb_weights", p, 850.0, w) == cb.CB_ERR_HISTORY_NOT_FULL
+    slot_t, head, count = cb.cb_plan_history(p, 3)
+    assert (head, count) == (0, 0)
+    assert cb.cb_plan_num_groups(p) == 1
+    cb.cb_plan_destroy(p)
+
+
+def test_failed_launch_leaves_history_unchanged(cb):
+    torch = pytest.importorskip("torch")
+    if torch.cuda.is_available():
+        pytest.skip("needs a machine without a GPU (the push must fail at the CUDA call)")
+    p = cb.cb_plan_create([999.0, 900.0], 2, _tensors([64]), cb.CB_BF16, 0.0, 999.0)
+    cb.cb_plan_bind_cache(p, 0x100000, cb.cb_plan_cache_bytes(p))
+    rc = cb.raw_status("cb_cache_push", p, (ctypes.c_void_p * 1)(0x1000), 0, 999.0, None)
+    assert rc == cb.CB_ERR_CUDA
+    assert cb.cb_last_error_message() != ""
+    assert cb.cb_plan_history(p, 2)[2] == 0
+    cb.cb_plan_destroy(p)
+
+
+def _workload_nodes(w, orc):
+    mask = orc.full_schedule(w.T, w.r, w.s0, w.s1, w.K)
+    ts = np.array(w.timesteps)
+    return ts[mask], ts[~mask]
+
+
+@pytest.mark.parametrize("name", ["dit256", "dit256-k3", "dit512", "pixart", "flux"])
+def test_exported_weight_table_matches_oracle(cb, orc, name):
+    """The prepackaged table (Alg. 1 offline stage) for every skipped step of the
+    schedule, against the oracle's Lagrange basis on the same K preceding nodes."""
+    from paper_2608_23429_gb300 import workloads
+    w = workloads.PRESETS[name]()
+    nodes, targets = _workload_nodes(w, orc)
+    p = cb.cb_plan_create(nodes, w.K, [(0, 0, 8, -1)], cb.CB_BF16, w.t_min, w.t_max)
+    table = cb.cb_plan_export_weights(p, targets, w.K)
+    for t, row in zip(targets, table):
+        prev = nodes[nodes > t][-w.K:]  # timesteps decrease along the sampling order
+        ref = orc.weights(prev, t, w.t_min, w.t_max)
+        assert np.max(np.abs(row - ref)) <= 1e-12 * np.abs(ref).sum(), (name, t)
+    cb.cb_plan_destroy(p)
+
+
+def test_export_weights_edge_cases(cb, orc):
+    p = cb.cb_plan_create([900.0, 800.0, 700.0, 600.0], 4, [(0, 0, 8, -1)], cb.CB_FP32, 0.0, 1000.0)
+    tab = cb.cb_plan_export_weights(p, [575.0, 550.0, 500.0], 4)
+    assert np.allclose(tab[2], [-1, 4, -6, 4], rtol=0, atol=1e-13)  # one spacing past the newest node
+    with pytest.raises(cb.CbError) as e:
+        cb.cb_plan_export_weights(p, [650.0], 4)  # only 3 nodes precede it
+    assert e.value.status == cb.CB_ERR_HISTORY_NOT_FULL
+    cb.cb_plan_destroy(p)
