@@ -33,7 +33,8 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "extrapolation GB/s & % of HBM peak; µs per skipped step (all blocks), 1 GB300"
-KERNEL_SOURCES = ["paper_2608_23429_gb300/csrc/extrapolate.cu", "paper_2608_23429_gb300/csrc/cb_device.h"]
+KERNEL_SOURCES = ["paper_2608_23429_gb300/csrc/extrapolate_bulk.cu", "paper_2608_23429_gb300/csrc/extrapolate.cu",
+                  "paper_2608_23429_gb300/csrc/cb_math.cuh", "paper_2608_23429_gb300/csrc/cb_device.h"]
 
 
 def kernel_hash() -> str:
@@ -55,7 +56,7 @@ def measured_peaks() -> tuple[float, str]:
 def recorded_traffic(config: str) -> float | None:
     """DRAM bytes per launch from the committed ncu summary, if it was taken on
     the current kernel source (else None)."""
-    path = os.path.join(ROOT, "profiles", f"extrapolate_{config}_traffic.txt")
+    path = os.path.join(ROOT, "profiles", f"extrapolate_bulk_{config}_traffic.txt")
     try:
         fields = dict(line.split("=", 1) for line in open(path).read().split() if "=" in line)
     except OSError:
@@ -265,6 +266,8 @@ def run_ours(args):
     plan = cb.cb_plan_create(node_t, K, tensors, cdt, w.t_min, w.t_max)
     cache = torch.empty(cb.cb_plan_cache_bytes(plan), dtype=torch.uint8, device=dev)
     cb.cb_plan_bind_cache(plan, cache, cache.numel())
+    cb.cb_plan_set_option(plan, cb.CB_OPT_KERNEL, {"auto": cb.CB_KERNEL_AUTO, "direct": cb.CB_KERNEL_DIRECT,
+                                                   "bulk": cb.CB_KERNEL_BULK}[args.kernel])
     stream = torch.cuda.Stream(device=dev)
     for s in pushed:  # full steps of the schedule up to the timed window
         feats = [wl.trajectory(w, i, w.timesteps[s], s, dev) for i in range(len(w.tensors))]
@@ -302,6 +305,9 @@ def run_ours(args):
         if ws > 1:
             dist.barrier()
     clocks = clk.summary()
+    dev_status = cb.cb_plan_device_status(plan, stream=stream)
+    if dev_status != 0:
+        raise RuntimeError(f"device status {dev_status}: a bounded wait ran out during the timed steps")
     total_ms = t_all0.elapsed_time(t_all1)
     kern_ms = [a.elapsed_time(b) for a, b in ev]
     total_ms = max_over_ranks(total_ms, dev)
@@ -342,7 +348,8 @@ def run_ours(args):
             "roofline": {"bound": "hbm", "achieved": round(achieved, 2), "peak": peak, "unit": "GB/s",
                          "frac": round(achieved / peak, 4), "peak_source": peak_src,
                          "traffic": recorded_traffic(args.config) if args.scale == 1 else None,
-                         "kernel": "extrapolate_kernel", "avg_launch_us": round(avg_kern * 1e3, 2)},
+                         "kernel": "extrapolate_kernel" if args.kernel == "direct" else "extrapolate_bulk_kernel",
+                         "avg_launch_us": round(avg_kern * 1e3, 2)},
             "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks, "gpu_launches": args.steps,
         }
         print(json.dumps(line))
@@ -398,6 +405,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--config", default="flux", choices=["dit256", "dit256-k3", "dit512", "pixart", "flux"])
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--kernel", default="auto", choices=["auto", "direct", "bulk"],
+                    help="skipped-step kernel variant (both compute identical bits)")
     ap.add_argument("--scale", type=int, default=1,
                     help="divide every tensor's token count (small cases for profiling only)")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)

@@ -50,6 +50,7 @@ extern "C" {
 #define CB_MAX_TENSORS 256    /* branch tensors per plan */
 #define CB_MAX_BRANCHES 4     /* branch tensors sharing one residual group */
 #define CB_CACHE_ALIGN 256    /* byte alignment of the cache arena and of each tensor in it */
+#define CB_STATUS_BYTES 256   /* device status block at the end of the cache arena */
 
 typedef struct cb_plan cb_plan; /* opaque, host-owned */
 
@@ -80,6 +81,23 @@ enum {
     CB_ERR_LIMIT = -8              /* a size beyond CB_MAX_K / CB_MAX_TENSORS / CB_MAX_BRANCHES */
 };
 
+/* Options of cb_plan_set_option. */
+enum {
+    CB_OPT_KERNEL = 1,  /* skipped-step kernel: CB_KERNEL_AUTO (default), _DIRECT or _BULK */
+    CB_OPT_WAIT_NS = 2, /* limit of every device-side wait of the bulk kernel, ns (default 1e9) */
+    CB_OPT_TEST_WITHHOLD = 3 /* 1: (tests of the failure path only) the bulk kernel's producer
+                                announces each CTA's first unit but never issues its copies, so
+                                that the consumers' wait runs out; outputs are then invalid */
+};
+enum { CB_KERNEL_AUTO = 0, CB_KERNEL_DIRECT = 1, CB_KERNEL_BULK = 2 };
+
+/* Codes OR-ed into the device status word (cb_plan_device_status). */
+enum {
+    CB_DEV_CONSUMER_TIMEOUT = 1, /* a consumer's wait for a filled stage ran out */
+    CB_DEV_PRODUCER_TIMEOUT = 2, /* the producer's wait for a released stage ran out */
+    CB_DEV_DRAIN_TIMEOUT = 4     /* the producer's final wait for its own copies ran out */
+};
+
 /* Full-computation schedule (Sec. 3.3, Eq. for F; Alg. 1 offline stage):
  *   s in F  iff  s not in [s0, T-1-s1]  or  r divides (s - s0),   s in [0, T-1],
  * then, when K > 0, every step whose history would hold fewer than K entries
@@ -102,8 +120,9 @@ int cb_schedule_full(int T, int r, int s0, int s1, int K, uint8_t* is_full, int*
 int cb_plan_create(const double* node_t, int n_nodes, int K, const cb_tensor_desc* tensors,
                    int n_tensors, cb_dtype cache_dtype, double t_min, double t_max, cb_plan** out);
 
-/* Bytes of device memory the history buffer needs: K slots, each holding every
- * tensor at a CB_CACHE_ALIGN-aligned offset. */
+/* Bytes of device memory the history buffer needs: K slots followed by a
+ * CB_STATUS_BYTES status block. Slot p starts at p * slot_bytes; inside it
+ * tensor i starts at sum_{k<i} roundup(numel_k * esize, CB_CACHE_ALIGN). */
 size_t cb_plan_cache_bytes(const cb_plan* plan);
 
 /* Attach caller-owned device memory as the history buffer (the plan never
@@ -170,6 +189,22 @@ int cb_plan_export_weights(const cb_plan* plan, const double* targets, int n_tar
  * head the slot of the oldest entry, count the number of entries (<= K).
  * Any output pointer may be NULL. */
 int cb_plan_history(const cb_plan* plan, double* slot_t, int* head, int* count);
+
+/* Set a plan option (CB_OPT_*). CB_OPT_KERNEL selects the skipped-step
+ * kernel: the direct-load kernel (each thread loads its K vectors from HBM) or
+ * the bulk-copy pipeline (a producer warp stages the K chunks of each tile in
+ * shared memory with cp.async.bulk; CTAs of 544 threads, one per SM); both
+ * compute identical bits. CB_OPT_WAIT_NS bounds every wait of the bulk kernel
+ * on a shared-memory barrier; a wait that runs out makes the kernel record a
+ * CB_DEV_* code in the device status word and return early (its outputs are
+ * then incomplete). Errors: CB_ERR_ARG. */
+int cb_plan_set_option(cb_plan* plan, int option, int64_t value);
+
+/* Read the device status word into *status (0 = no device-side event since
+ * the last read) and clear it. Enqueues a 4-byte copy and a 4-byte memset on
+ * `stream` and synchronises that stream. Errors: CB_ERR_ARG, CB_ERR_UNBOUND,
+ * CB_ERR_CUDA. */
+int cb_plan_device_status(cb_plan* plan, int* status, void* stream);
 
 /* Empty H (a new sample starts). */
 int cb_plan_reset(cb_plan* plan);

@@ -20,7 +20,7 @@ LIB = os.path.join(HERE, "libchebboost.so")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["extrapolate.cu", "push.cu", "plan.cpp"]
+SOURCES = ["extrapolate.cu", "extrapolate_bulk.cu", "push.cu", "plan.cpp"]
 
 
 def _nvcc() -> str:
@@ -44,7 +44,7 @@ def _stale(target: str, deps: list[str]) -> bool:
 def build(force: bool = False, verbose: bool = False) -> str:
     nvcc = _nvcc()
     os.makedirs(BUILD, exist_ok=True)
-    headers = [os.path.join(CSRC, h) for h in os.listdir(CSRC) if h.endswith(".h")]
+    headers = [os.path.join(CSRC, h) for h in os.listdir(CSRC) if h.endswith((".h", ".cuh"))]
     headers.append(os.path.join(INCLUDE, "chebboost.h"))
     objs, jobs = [], []
     for src in SOURCES:

@@ -24,7 +24,10 @@ if not os.path.exists(LIB_PATH):
 _lib = ctypes.CDLL(LIB_PATH)
 
 CB_BF16, CB_FP32 = 0, 1
-CB_MAX_K, CB_MAX_TENSORS, CB_MAX_BRANCHES, CB_CACHE_ALIGN = 8, 256, 4, 256
+CB_MAX_K, CB_MAX_TENSORS, CB_MAX_BRANCHES, CB_CACHE_ALIGN, CB_STATUS_BYTES = 8, 256, 4, 256, 256
+CB_OPT_KERNEL, CB_OPT_WAIT_NS, CB_OPT_TEST_WITHHOLD = 1, 2, 3
+CB_KERNEL_AUTO, CB_KERNEL_DIRECT, CB_KERNEL_BULK = 0, 1, 2
+CB_DEV_CONSUMER_TIMEOUT, CB_DEV_PRODUCER_TIMEOUT, CB_DEV_DRAIN_TIMEOUT = 1, 2, 4
 CB_OK, CB_ERR_ARG, CB_ERR_ALIGN, CB_ERR_NODES_DEGENERATE = 0, -1, -2, -3
 CB_ERR_HISTORY_NOT_FULL, CB_ERR_ORDER, CB_ERR_UNBOUND, CB_ERR_CUDA, CB_ERR_LIMIT = -4, -5, -6, -7, -8
 
@@ -48,6 +51,8 @@ _sig = {
     "cb_plan_export_weights": ([_P, _P, _I, _P], _I),
     "cb_plan_history": ([_P, _P, _P, _P], _I),
     "cb_plan_reset": ([_P], _I),
+    "cb_plan_set_option": ([_P, _I, ctypes.c_int64], _I),
+    "cb_plan_device_status": ([_P, _P, _P], _I),
     "cb_plan_num_groups": ([_P], _I),
     "cb_plan_destroy": ([_P], None),
     "cb_status_string": ([_I], ctypes.c_char_p),
@@ -170,6 +175,16 @@ def cb_plan_history(plan, K: int):
 
 def cb_plan_reset(plan) -> None:
     _check(_lib.cb_plan_reset(plan), "cb_plan_reset")
+
+
+def cb_plan_set_option(plan, option: int, value: int) -> None:
+    _check(_lib.cb_plan_set_option(plan, option, int(value)), "cb_plan_set_option")
+
+
+def cb_plan_device_status(plan, stream=None) -> int:
+    st = ctypes.c_int(0)
+    _check(_lib.cb_plan_device_status(plan, ctypes.byref(st), _stream(stream)), "cb_plan_device_status")
+    return st.value
 
 
 def cb_plan_num_groups(plan) -> int:

@@ -35,6 +35,10 @@ struct ExtrapArgs {
     int out_bf16;    // predictions are bf16 (else fp32)
     int resid_bf16;  // hidden states are bf16 (else fp32)
     int precise;     // 1: compensated (Dot2) arithmetic for every element
+    int stages;                  // bulk variant: shared-memory pipeline depth
+    unsigned long long wait_ns;  // bulk variant: limit of every barrier wait
+    int* status;                 // bulk variant: device status word (codes OR-ed in)
+    int withhold_first;          // bulk variant, tests only: announce but never issue the first copies
     int tile_begin[kMaxItems + 1];
     long long numel[kMaxItems];
     void* resid[kMaxItems];           // hidden state of the item, or null
@@ -61,6 +65,13 @@ constexpr long long push_tile_elems = (long long)kThreads * 2 * kVecElems;
 
 cudaError_t launch_extrapolate(const ExtrapArgs& a, int K, bool cache_bf16, int grid, cudaStream_t s);
 cudaError_t extrapolate_blocks_per_sm(int K, bool cache_bf16, int* blocks);
+
+// Bulk-copy pipeline variant (extrapolate_bulk.cu).
+size_t bulk_smem_bytes(int K, int stages);
+int bulk_threads();
+cudaError_t prepare_extrapolate_bulk(int K, bool cache_bf16, size_t smem);
+cudaError_t launch_extrapolate_bulk(const ExtrapArgs& a, int K, bool cache_bf16, int grid, size_t smem,
+                                    cudaStream_t s);
 
 cudaError_t launch_push(const PushArgs& a, bool src_bf16, bool dst_bf16, int grid, cudaStream_t s);
 cudaError_t push_blocks_per_sm(bool src_bf16, bool dst_bf16, int* blocks);

@@ -1,0 +1,385 @@
+// Internal: the per-element arithmetic of the skipped-step kernels, shared by
+// the direct-load kernel (extrapolate.cu) and the bulk-copy pipeline kernel
+// (extrapolate_bulk.cu) so that both produce identical bits.
+//
+// Fast path. s = sum_j w_hi[j] F_j by fp32 FMA and, alongside,
+// a = sum_j |w_hi[j]| |F_j|. With u = 2^-24 the FMA chain plus the dropped low
+// half of each weight give |s - P| <= (K+1) u a (1 + O(Ku)). Whenever
+// (K+2) u a (1.01) <= 2^-9 |s| that error is below the smallest bf16 spacing
+// next to s, so bf16(s) lies within one bf16 ulp of bf16(P) (guard_ok).
+// Elements failing the test (strong cancellation, ~1e-4..3e-3 of them) are
+// recomputed from the values already loaded with Dot2 (Ogita, Rump &
+// Oishi, "Accurate Sum and Dot Product", SIAM J. Sci. Comput. 26(6), 2005:
+// TwoProduct by FMA plus TwoSum) with the weights as fp32 pairs hi + lo, and
+// the unevaluated result pair is rounded once. fp32 results always take Dot2.
+#pragma once
+
+#include <cuda_bf16.h>
+
+#include "cb_device.h"
+
+namespace cbk {
+namespace {
+
+constexpr float kU = 0x1.0p-24f;
+
+__device__ __forceinline__ uint4 ld_stream(const unsigned char* p) {
+    uint4 v;
+    asm("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+        : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+        : "l"(p));
+    return v;
+}
+
+__device__ __forceinline__ void unpack_bf16x8(const uint4& v, float (&f)[8]) {
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        f[2 * i] = __uint_as_float(w[i] << 16);
+        f[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+    }
+}
+
+__device__ __forceinline__ void unpack_f32x8(const uint4& a, const uint4& b, float (&f)[8]) {
+    f[0] = __uint_as_float(a.x); f[1] = __uint_as_float(a.y);
+    f[2] = __uint_as_float(a.z); f[3] = __uint_as_float(a.w);
+    f[4] = __uint_as_float(b.x); f[5] = __uint_as_float(b.y);
+    f[6] = __uint_as_float(b.z); f[7] = __uint_as_float(b.w);
+}
+
+template <bool CB16>
+__device__ __forceinline__ void unpack(const uint4 (&r)[CB16 ? 1 : 2], float (&f)[8]) {
+    if constexpr (CB16)
+        unpack_bf16x8(r[0], f);
+    else
+        unpack_f32x8(r[0], r[CB16 ? 0 : 1], f);
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);  // RNE; .x is the low half
+    return *reinterpret_cast<uint32_t*>(&h);
+}
+
+__device__ __forceinline__ uint16_t bf16_bits(float x) { return __bfloat16_as_ushort(__float2bfloat16_rn(x)); }
+
+// ---- error-free transformations (explicitly rounded operations, never contracted)
+__device__ __forceinline__ void two_sum(float a, float b, float& s, float& e) {
+    s = __fadd_rn(a, b);
+    const float bb = __fsub_rn(s, a);
+    e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+}
+
+// One Dot2 term: (p, c) += (w_hi + w_lo) * f, p the running sum, c its error.
+__device__ __forceinline__ void dot2_step(float w_hi, float w_lo, float f, float& p, float& c) {
+    const float h = __fmul_rn(w_hi, f);
+    const float r = __fmaf_rn(w_hi, f, -h);  // exact: w_hi*f - h
+    float q;
+    two_sum(p, h, p, q);
+    c = __fadd_rn(c, __fadd_rn(q, r));
+    c = __fmaf_rn(w_lo, f, c);
+}
+
+// bf16 of the exact value hi + lo, where hi = fl(hi + lo) (so |lo| <= ulp(hi)/2).
+// Only when hi sits exactly on a bf16 rounding midpoint can lo change the
+// outcome; then the sign of lo decides, otherwise hi rounds like hi + lo.
+__device__ __forceinline__ uint16_t bf16_of_pair(float hi, float lo) {
+    const uint32_t b = __float_as_uint(hi);
+    if ((b & 0xFFFFu) == 0x8000u && lo != 0.0f && (b & 0x7F800000u) != 0x7F800000u) {
+        const bool away = (lo > 0.0f) == (hi > 0.0f);
+        return (uint16_t)((b >> 16) + (away ? 1u : 0u));
+    }
+    return bf16_bits(hi);
+}
+
+template <bool CB16>
+__device__ __forceinline__ float load_cache_elem(const unsigned char* base, long long e) {
+    if constexpr (CB16) {
+        const uint16_t h = reinterpret_cast<const uint16_t*>(base)[e];
+        return __uint_as_float((uint32_t)h << 16);
+    } else {
+        return reinterpret_cast<const float*>(base)[e];
+    }
+}
+
+__device__ __forceinline__ float load_elem(const void* p, bool bf16, long long e) {
+    if (bf16) return __uint_as_float((uint32_t)(reinterpret_cast<const uint16_t*>(p)[e]) << 16);
+    return reinterpret_cast<const float*>(p)[e];
+}
+
+__device__ __forceinline__ void store_pair(void* p, bool bf16, long long e, float hi, float lo) {
+    if (bf16)
+        reinterpret_cast<uint16_t*>(p)[e] = bf16_of_pair(hi, lo);
+    else
+        reinterpret_cast<float*>(p)[e] = hi;
+}
+
+// Compensated value of member tensor (byte offset moff) at element e.
+template <bool CB16>
+__device__ __noinline__ void exact_member(const ExtrapArgs& A, int K, long long moff, long long e, float& hi,
+                                          float& lo) {
+    float p = 0.0f, c = 0.0f;
+    for (int j = 0; j < K; ++j) {
+        const float f = load_cache_elem<CB16>(A.cache + A.slot_off[j] + moff, e);
+        dot2_step(A.w_hi[j], A.w_lo[j], f, p, c);
+    }
+    two_sum(p, c, hi, lo);
+}
+
+// Compensated hidden-state update of item `it` at element e: x + sum_b P_b.
+template <bool CB16>
+__device__ __noinline__ void exact_resid(const ExtrapArgs& A, int K, int it, long long e, float x, float& hi,
+                                         float& lo) {
+    float tp = x, tc = 0.0f;
+    const int first = A.first[it];
+    for (int m = 0; m < A.nb[it]; ++m) {
+        float h, l, q;
+        exact_member<CB16>(A, K, A.m_off[first + m], e, h, l);
+        two_sum(tp, h, tp, q);
+        tc = __fadd_rn(tc, __fadd_rn(q, l));
+    }
+    two_sum(tp, tc, hi, lo);
+}
+
+// One element of item `it` through the compensated path, every member and the
+// hidden state (misaligned items and ragged tails).
+template <bool CB16>
+__device__ __noinline__ void scalar_element(const ExtrapArgs& A, int K, int it, long long e) {
+    const int first = A.first[it];
+    void* resid = A.resid[it];
+    float tp = 0.0f, tc = 0.0f;
+    for (int m = 0; m < A.nb[it]; ++m) {
+        float hi, lo, q;
+        exact_member<CB16>(A, K, A.m_off[first + m], e, hi, lo);
+        if (A.m_out[first + m]) store_pair(A.m_out[first + m], A.out_bf16, e, hi, lo);
+        two_sum(tp, hi, tp, q);
+        tc = __fadd_rn(tc, __fadd_rn(q, lo));
+    }
+    if (resid) {
+        float q, hi, lo;
+        two_sum(tp, load_elem(resid, A.resid_bf16, e), tp, q);
+        tc = __fadd_rn(tc, q);
+        two_sum(tp, tc, hi, lo);
+        store_pair(resid, A.resid_bf16, e, hi, lo);
+    }
+}
+
+__device__ __forceinline__ void load_x8(const void* p, bool bf16, long long e, float (&x)[8]) {
+    if (bf16) {
+        const uint4 v = *reinterpret_cast<const uint4*>(reinterpret_cast<const uint16_t*>(p) + e);
+        unpack_bf16x8(v, x);
+    } else {
+        const uint4* q = reinterpret_cast<const uint4*>(reinterpret_cast<const float*>(p) + e);
+        unpack_f32x8(q[0], q[1], x);
+    }
+}
+
+__device__ __forceinline__ void store_bf16x8(void* p, long long e, const uint32_t (&pk)[4]) {
+    *reinterpret_cast<uint4*>(reinterpret_cast<uint16_t*>(p) + e) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+}
+
+__device__ __forceinline__ void store_f32x8(void* p, long long e, const float (&v)[8]) {
+    uint4* q = reinterpret_cast<uint4*>(reinterpret_cast<float*>(p) + e);
+    q[0] = make_uint4(__float_as_uint(v[0]), __float_as_uint(v[1]), __float_as_uint(v[2]), __float_as_uint(v[3]));
+    q[1] = make_uint4(__float_as_uint(v[4]), __float_as_uint(v[5]), __float_as_uint(v[6]), __float_as_uint(v[7]));
+}
+
+__device__ __forceinline__ void set_half(uint32_t (&pk)[4], int e, uint16_t h) {
+    uint32_t& w = pk[e >> 1];
+    w = (e & 1) ? ((w & 0x0000FFFFu) | ((uint32_t)h << 16)) : ((w & 0xFFFF0000u) | h);
+}
+
+// Running sums of one item across its members (the fused hidden-state update):
+// fast path x = sum_b s_b, y = sum_b a_b; compensated path x + y is the
+// unevaluated sum (running value and its error).
+template <int UV>
+struct Acc {
+    float x[UV][8];
+    float y[UV][8];
+    __device__ __forceinline__ void zero() {
+#pragma unroll
+        for (int u = 0; u < UV; ++u)
+#pragma unroll
+            for (int e = 0; e < 8; ++e) x[u][e] = y[u][e] = 0.0f;
+    }
+};
+
+template <int K, bool CB16, int UV>
+using RawVecs = uint4[UV][K][CB16 ? 1 : 2];
+
+// Dot2 value of element e of vector u from its K history values as loaded
+// (registers or shared memory); used where the fast path's guard fails.
+template <int K, bool CB16, int UV>
+__device__ __forceinline__ void exact_from_raw(const ExtrapArgs& A, const RawVecs<K, CB16, UV>& raw, int u, int e,
+                                               float& hi, float& lo) {
+    float p = 0.0f, c = 0.0f;
+#pragma unroll
+    for (int j = 0; j < K; ++j) {
+        float f[8];
+        unpack<CB16>(raw[u][j], f);
+        float fe = f[0];
+#pragma unroll
+        for (int i = 1; i < 8; ++i) fe = (e == i) ? f[i] : fe;
+        dot2_step(A.w_hi[j], A.w_lo[j], fe, p, c);
+    }
+    two_sum(p, c, hi, lo);
+}
+
+// Fast-path guard: with |s - P| <= (K+1) u a (1 + O(Ku)), the test
+// (K+2) u a (1.01) <= 2^-9 |s| keeps the interval between s and P shorter than
+// the smallest bf16 spacing next to s (2^-8 |s| in s's binade, 2^-9 |s| below
+// it), so it holds at most one rounding midpoint and bf16(s) is within one ulp
+// of bf16(P).
+__device__ __forceinline__ bool guard_ok(float g, float a, float s) { return g * a <= 0x1.0p-9f * fabsf(s); }
+
+// Fast path for one member over UV aligned 8-element vectors already loaded
+// into registers: bf16 prediction (if out) and accumulation into acc. The
+// rare guarded elements are recomputed from the loaded values (FROM_RAW: no
+// memory latency, but the values stay live and cost registers) or re-read
+// from global memory (member byte offset moff).
+template <int K, bool CB16, int UV, bool FROM_RAW>
+__device__ __forceinline__ void member_fast(const ExtrapArgs& A, long long moff, void* out,
+                                            const long long (&ev)[UV], const RawVecs<K, CB16, UV>& raw,
+                                            bool accumulate, Acc<UV>& acc) {
+    const float g_out = (float)(K + 2) * kU * 1.01f;
+#pragma unroll
+    for (int u = 0; u < UV; ++u) {
+        float s[8], a[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) s[e] = a[e] = 0.0f;
+#pragma unroll
+        for (int j = 0; j < K; ++j) {
+            float f[8];
+            unpack<CB16>(raw[u][j], f);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                s[e] = fmaf(A.w_hi[j], f[e], s[e]);
+                a[e] = fmaf(A.w_abs[j], fabsf(f[e]), a[e]);
+            }
+        }
+        if (out) {
+            uint32_t pk[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) pk[i] = pack_bf16x2(s[2 * i], s[2 * i + 1]);
+            unsigned bad = 0;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) bad |= guard_ok(g_out, a[e], s[e]) ? 0u : (1u << e);
+            while (bad) {  // rare: recompute the failing elements with Dot2
+                const int e = __ffs(bad) - 1;
+                bad &= bad - 1;
+                float hi, lo;
+                if constexpr (FROM_RAW)
+                    exact_from_raw<K, CB16, UV>(A, raw, u, e, hi, lo);
+                else
+                    exact_member<CB16>(A, K, moff, ev[u] + e, hi, lo);
+                set_half(pk, e, bf16_of_pair(hi, lo));
+            }
+            store_bf16x8(out, ev[u], pk);
+        }
+        if (accumulate) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                acc.x[u][e] += s[e];
+                acc.y[u][e] += a[e];
+            }
+        }
+    }
+}
+
+// Fast path: hidden state <- bf16(x + sum_b s_b), guarded like the members.
+template <int K, bool CB16, int UV>
+__device__ __forceinline__ void resid_fast(const ExtrapArgs& A, int it, const long long (&ev)[UV],
+                                           const Acc<UV>& acc, void* resid) {
+    const float g_res = (float)(K + A.nb[it] + 3) * kU * 1.01f;
+#pragma unroll
+    for (int u = 0; u < UV; ++u) {
+        float x[8], t[8];
+        uint32_t pk[4];
+        load_x8(resid, true, ev[u], x);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) t[e] = acc.x[u][e] + x[e];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) pk[i] = pack_bf16x2(t[2 * i], t[2 * i + 1]);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            if (!guard_ok(g_res, acc.y[u][e] + fabsf(x[e]), t[e])) {
+                float hi, lo;
+                exact_resid<CB16>(A, K, it, ev[u] + e, x[e], hi, lo);
+                set_half(pk, e, bf16_of_pair(hi, lo));
+            }
+        }
+        store_bf16x8(resid, ev[u], pk);
+    }
+}
+
+// Compensated path for one member (any fp32 prediction or hidden state).
+template <int K, bool CB16, int UV>
+__device__ __forceinline__ void member_precise(const ExtrapArgs& A, void* out, const long long (&ev)[UV],
+                                               const RawVecs<K, CB16, UV>& raw, bool accumulate,
+                                               Acc<UV>& acc) {
+#pragma unroll
+    for (int u = 0; u < UV; ++u) {
+        float p[8], c[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) p[e] = c[e] = 0.0f;
+#pragma unroll
+        for (int j = 0; j < K; ++j) {
+            float f[8];
+            unpack<CB16>(raw[u][j], f);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) dot2_step(A.w_hi[j], A.w_lo[j], f[e], p[e], c[e]);
+        }
+        float hi[8], lo[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) two_sum(p[e], c[e], hi[e], lo[e]);
+        if (out) {
+            if (A.out_bf16) {
+                uint32_t pk[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                    pk[i] = (uint32_t)bf16_of_pair(hi[2 * i], lo[2 * i]) |
+                            ((uint32_t)bf16_of_pair(hi[2 * i + 1], lo[2 * i + 1]) << 16);
+                store_bf16x8(out, ev[u], pk);
+            } else {
+                store_f32x8(out, ev[u], hi);
+            }
+        }
+        if (accumulate) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                float q;
+                two_sum(acc.x[u][e], hi[e], acc.x[u][e], q);
+                acc.y[u][e] = __fadd_rn(acc.y[u][e], __fadd_rn(q, lo[e]));
+            }
+        }
+    }
+}
+
+template <int UV>
+__device__ __forceinline__ void resid_precise(const ExtrapArgs& A, const long long (&ev)[UV], Acc<UV>& acc,
+                                              void* resid) {
+#pragma unroll
+    for (int u = 0; u < UV; ++u) {
+        float x[8], hi[8], lo[8];
+        load_x8(resid, A.resid_bf16, ev[u], x);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            float q;
+            two_sum(acc.x[u][e], x[e], acc.x[u][e], q);
+            acc.y[u][e] = __fadd_rn(acc.y[u][e], q);
+            two_sum(acc.x[u][e], acc.y[u][e], hi[e], lo[e]);
+        }
+        if (A.resid_bf16) {
+            uint32_t pk[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                pk[i] = (uint32_t)bf16_of_pair(hi[2 * i], lo[2 * i]) |
+                        ((uint32_t)bf16_of_pair(hi[2 * i + 1], lo[2 * i + 1]) << 16);
+            store_bf16x8(resid, ev[u], pk);
+        } else {
+            store_f32x8(resid, ev[u], hi);
+        }
+    }
+}
+
+}  // namespace
+}  // namespace cbk

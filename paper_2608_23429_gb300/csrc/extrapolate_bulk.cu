@@ -1,0 +1,265 @@
+// Skipped-step kernel, bulk-copy pipeline variant (same arithmetic and bits as
+// extrapolate.cu; Sec. 3.3, Eq. for f_t; Alg. 1, extrapolation branch).
+//
+// One CTA per SM. A producer warp moves, for every work unit (one tile of one
+// branch tensor), the K history chunks of 8 KB each from HBM into a ring of
+// shared-memory stages with cp.async.bulk (the Blackwell bulk-copy engine),
+// each stage guarded by a "full" mbarrier (transaction bytes) and an "empty"
+// mbarrier (consumer warps). Eight consumer warps read their two 8-element
+// vectors of the K chunks from shared memory (the same element-to-thread map
+// as the direct kernel), release the stage, and compute and store from
+// registers. Nine warps leave each thread up to 168 registers. With S stages of K x 8 KB (S = 5 for K = 5) up to
+// ~160 KB per SM stay in flight independently of the consumers' register use,
+// which is what bounds the direct-load variant.
+//
+// Every wait is bounded (%globaltimer). A wait that runs out records a code in
+// the plan's device status word and the thread returns; the producer then
+// waits, with its own limit (at least 10 ms), for the copies it has issued
+// before it exits. A test option makes the producer announce the first unit's
+// bytes without issuing its copies, so that the consumers' wait runs out with
+// no fault and nothing in flight.
+#include "cb_math.cuh"
+
+namespace cbk {
+namespace {
+
+constexpr int kConsumerWarps = 8;
+constexpr int kBulkThreads = (kConsumerWarps + 1) * 32;
+constexpr int kChunkBytes = 8192;   // one history entry's share of a tile
+constexpr int kBarrierBytes = 256;  // full[S] and empty[S] barriers, S <= 16
+constexpr unsigned long long kMinDrainNs = 10000000ull;  // copies land in microseconds
+
+__device__ __forceinline__ uint32_t smem_addr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ unsigned long long now_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Wait for the phase with the given parity to complete, for at most limit_ns.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, unsigned long long limit_ns) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = now_ns();
+    while (!mbar_try_wait(bar, parity))
+        if (now_ns() - t0 > limit_ns) return false;
+    return true;
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+
+// Global -> shared bulk copy completing `bytes` transaction bytes on `bar`.
+// dst, src 16-byte aligned; bytes a multiple of 16.
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     dst),
+                 "l"(src), "r"(bytes), "r"(bar)
+                 : "memory");
+}
+
+__device__ __forceinline__ void record(int* status, int code) {
+    if (status) atomicOr(status, code);
+}
+
+template <int K, bool CB16>
+__global__ void __launch_bounds__(kBulkThreads, 1) extrapolate_bulk_kernel(const __grid_constant__ ExtrapArgs A) {
+    extern __shared__ __align__(128) unsigned char smem[];
+    constexpr long long TE = tile_elems(CB16);  // 8 KB per history chunk for both cache types
+    constexpr int ES = CB16 ? 2 : 4;
+    constexpr int U = vectors_per_thread(CB16);  // vectors per consumer thread per tile
+    static_assert(kConsumerWarps * 32 == kThreads, "consumers use the direct kernel's thread map");
+    static_assert(TE * ES == kChunkBytes, "one tile of one history entry is one chunk");
+    const int S = A.stages;
+    const uint32_t full0 = smem_addr(smem);
+    const uint32_t empty0 = full0 + 8u * (uint32_t)S;
+    const uint32_t buf0 = smem_addr(smem + kBarrierBytes);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(full0 + 8u * s, 1);
+            mbar_init(empty0 + 8u * s, kConsumerWarps);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncthreads();
+
+    if (warp == kConsumerWarps) {  // ---------------------------------- producer
+        if (lane != 0) return;
+        int it = 0;
+        unsigned u = 0;
+        bool ok = true;
+        for (int tile = blockIdx.x; ok && tile < A.tiles_total; tile += gridDim.x) {
+            while (tile >= A.tile_begin[it + 1]) ++it;
+            const long long numel = A.numel[it];
+            const long long e0 = (long long)(tile - A.tile_begin[it]) * TE;
+            // consumers read shared memory only for whole tiles of aligned items;
+            // for the ragged last tile (or a misaligned item) the stage is
+            // cycled without data and they recompute from global memory
+            const bool full_tile = A.vec_ok[it] && e0 + TE <= numel;
+            const uint32_t bytes = full_tile ? (uint32_t)kChunkBytes : 0u;
+            const int first = A.first[it];
+            for (int m = 0; m < A.nb[it]; ++m, ++u) {
+                const uint32_t stage = u % (unsigned)S, q = u / (unsigned)S;
+                if (q > 0 && !mbar_wait(empty0 + 8u * stage, (q - 1) & 1u, A.wait_ns)) {
+                    record(A.status, 2);
+                    ok = false;
+                    break;
+                }
+                mbar_expect_tx(full0 + 8u * stage, (uint32_t)K * bytes);
+                if (bytes && !(A.withhold_first && u == 0)) {
+                    const unsigned char* src = A.cache + A.m_off[first + m] + e0 * ES;
+#pragma unroll
+                    for (int j = 0; j < K; ++j)
+                        bulk_g2s(buf0 + (stage * K + j) * (uint32_t)kChunkBytes, src + A.slot_off[j], bytes,
+                                 full0 + 8u * stage);
+                }
+            }
+        }
+        // never leave while copies into this CTA's shared memory are in flight
+        const unsigned long long drain_ns = A.wait_ns > kMinDrainNs ? A.wait_ns : kMinDrainNs;
+        for (unsigned q = u > (unsigned)S ? u - S : 0; q < u; ++q)
+            if (!mbar_wait(full0 + 8u * (q % S), (q / S) & 1u, drain_ns)) {
+                record(A.status, 4);
+                break;
+            }
+        return;
+    }
+
+    // ------------------------------------------------------------ consumers
+    const int c = threadIdx.x;
+    int it = 0;
+    unsigned u = 0;
+    for (int tile = blockIdx.x; tile < A.tiles_total; tile += gridDim.x) {
+        while (tile >= A.tile_begin[it + 1]) ++it;
+        const long long numel = A.numel[it];
+        const long long e0 = (long long)(tile - A.tile_begin[it]) * TE;
+        const int nb = A.nb[it];
+        const int first = A.first[it];
+        void* resid = A.resid[it];
+        // whole aligned tiles come from shared memory; the ragged last tile of a
+        // tensor and misaligned items take the compensated scalar path
+        const bool full_tile = A.vec_ok[it] && e0 + TE <= numel;
+        long long ev[U];
+#pragma unroll
+        for (int v = 0; v < U; ++v) ev[v] = e0 + ((long long)v * kThreads + c) * kVecElems;
+        Acc<U> acc;
+        acc.zero();
+        for (int m = 0; m < nb; ++m, ++u) {
+            const uint32_t stage = u % (unsigned)S, q = u / (unsigned)S;
+            if (!mbar_wait(full0 + 8u * stage, q & 1u, A.wait_ns)) {
+                record(A.status, 1);
+                return;
+            }
+            RawVecs<K, CB16, U> raw;
+            if (full_tile) {
+                const unsigned char* base = smem + kBarrierBytes + (size_t)stage * K * kChunkBytes;
+#pragma unroll
+                for (int v = 0; v < U; ++v)
+#pragma unroll
+                    for (int j = 0; j < K; ++j) {
+                        const unsigned char* p = base + (size_t)j * kChunkBytes + (size_t)(ev[v] - e0) * ES;
+                        raw[v][j][0] = *reinterpret_cast<const uint4*>(p);
+                        if constexpr (!CB16) raw[v][j][CB16 ? 0 : 1] = *reinterpret_cast<const uint4*>(p + 16);
+                    }
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(empty0 + 8u * stage);
+            if (full_tile) {
+                if (A.precise)
+                    member_precise<K, CB16, U>(A, A.m_out[first + m], ev, raw, resid != nullptr, acc);
+                else
+                    member_fast<K, CB16, U, true>(A, A.m_off[first + m], A.m_out[first + m], ev, raw,
+                                                  resid != nullptr, acc);
+            }
+        }
+        if (full_tile) {
+            if (resid) {
+                if (A.precise)
+                    resid_precise<U>(A, ev, acc, resid);
+                else
+                    resid_fast<K, CB16, U>(A, it, ev, acc, resid);
+            }
+        } else {
+            const long long end = e0 + TE < numel ? e0 + TE : numel;
+            for (long long e = e0 + c; e < end; e += kThreads) scalar_element<CB16>(A, K, it, e);
+        }
+    }
+}
+
+template <int K, bool CB16>
+cudaError_t launch_k(const ExtrapArgs& a, int grid, size_t smem, cudaStream_t s) {
+    extrapolate_bulk_kernel<K, CB16><<<grid, kBulkThreads, smem, s>>>(a);
+    return cudaGetLastError();
+}
+
+template <int K, bool CB16>
+cudaError_t prepare_k(size_t smem) {
+    return cudaFuncSetAttribute(extrapolate_bulk_kernel<K, CB16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)smem);
+}
+
+#define CB_K_SWITCH(K, CALL)                  \
+    switch (K) {                              \
+    case 1: return CALL(1);                   \
+    case 2: return CALL(2);                   \
+    case 3: return CALL(3);                   \
+    case 4: return CALL(4);                   \
+    case 5: return CALL(5);                   \
+    case 6: return CALL(6);                   \
+    case 7: return CALL(7);                   \
+    case 8: return CALL(8);                   \
+    default: return cudaErrorInvalidValue;    \
+    }
+
+}  // namespace
+
+size_t bulk_smem_bytes(int K, int stages) { return kBarrierBytes + (size_t)stages * K * kChunkBytes; }
+int bulk_threads() { return kBulkThreads; }
+
+cudaError_t prepare_extrapolate_bulk(int K, bool cache_bf16, size_t smem) {
+#define P_BF(k) prepare_k<k, true>(smem)
+#define P_F32(k) prepare_k<k, false>(smem)
+    if (cache_bf16) {
+        CB_K_SWITCH(K, P_BF)
+    }
+    CB_K_SWITCH(K, P_F32)
+#undef P_BF
+#undef P_F32
+}
+
+cudaError_t launch_extrapolate_bulk(const ExtrapArgs& a, int K, bool cache_bf16, int grid, size_t smem,
+                                    cudaStream_t s) {
+#define L_BF(k) launch_k<k, true>(a, grid, smem, s)
+#define L_F32(k) launch_k<k, false>(a, grid, smem, s)
+    if (cache_bf16) {
+        CB_K_SWITCH(K, L_BF)
+    }
+    CB_K_SWITCH(K, L_F32)
+#undef L_BF
+#undef L_F32
+}
+
+}  // namespace cbk

@@ -61,8 +61,10 @@ void coeff_of(const double* x, const double* rho, int n, double xq, double* w) {
 struct DeviceInfo {
     int device = -1;
     int sms = 0;
+    int smem_optin = 0;                    // largest dynamic shared memory per CTA
     int occ_extrap[2][CB_MAX_K + 1] = {};  // [cache_bf16][K]
     int occ_push[2][2] = {};               // [src_bf16][dst_bf16]
+    int bulk_stages[2][CB_MAX_K + 1] = {};  // pipeline depth once the kernel is prepared
 };
 
 }  // namespace
@@ -87,11 +89,16 @@ struct cb_plan {
     int count = 0;  // entries held (<= K)
     bool has_last = false;
     double last_t = 0;
+    bool status_clear = false;  // the device status word was zeroed since binding
+    int kernel = CB_KERNEL_AUTO;
+    unsigned long long wait_ns = 1000000000ull;
+    int withhold_first = 0;
     DeviceInfo dev;
     std::unique_ptr<cbk::ExtrapArgs> eargs{new cbk::ExtrapArgs};
     std::unique_ptr<cbk::PushArgs> pargs{new cbk::PushArgs};
 
     double tau(double t) const { return 2.0 * (t - t_min) / (t_max - t_min) - 1.0; }
+    int* status_word() const { return reinterpret_cast<int*>(cache + slot_bytes * (size_t)K); }
     int oldest() const { return count < K ? 0 : next; }
 };
 
@@ -105,6 +112,8 @@ int ensure_device(cb_plan* p) {
         DeviceInfo info;
         info.device = d;
         e = cudaDeviceGetAttribute(&info.sms, cudaDevAttrMultiProcessorCount, d);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
+        e = cudaDeviceGetAttribute(&info.smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, d);
         if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
         p->dev = info;
     }
@@ -122,6 +131,24 @@ int extrap_grid(cb_plan* p, int K, bool cb16, int tiles, int* grid) {
     }
     long long g = (long long)p->dev.sms * occ;
     *grid = (int)(tiles < g ? tiles : g);
+    return CB_OK;
+}
+
+// Pipeline depth of the bulk kernel: as many K x 8 KB stages as fit in one
+// CTA's shared memory (at most 8); the kernel's smem limit is raised once.
+int bulk_config(cb_plan* p, int K, bool cb16, int* stages, size_t* smem) {
+    int& st = p->dev.bulk_stages[cb16 ? 1 : 0][K];
+    if (st == 0) {
+        int s = 8;
+        while (s > 1 && cbk::bulk_smem_bytes(K, s) > (size_t)p->dev.smem_optin) --s;
+        if (cbk::bulk_smem_bytes(K, s) > (size_t)p->dev.smem_optin)
+            return cuda_fail(cudaErrorInvalidConfiguration, "bulk pipeline does not fit in shared memory");
+        cudaError_t e = cbk::prepare_extrapolate_bulk(K, cb16, cbk::bulk_smem_bytes(K, s));
+        if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute");
+        st = s;
+    }
+    *stages = st;
+    *smem = cbk::bulk_smem_bytes(K, st);
     return CB_OK;
 }
 
@@ -268,10 +295,22 @@ int run_extrapolate(cb_plan* p, const Window& win, double t_target, void* const*
 
     rc = ensure_device(p);
     if (rc != CB_OK) return rc;
-    int grid = 0;
-    rc = extrap_grid(p, p->K, cb16, (int)tiles, &grid);
+    if (p->kernel == CB_KERNEL_DIRECT) {
+        int grid = 0;
+        rc = extrap_grid(p, p->K, cb16, (int)tiles, &grid);
+        if (rc != CB_OK) return rc;
+        cudaError_t e = cbk::launch_extrapolate(A, p->K, cb16, grid, (cudaStream_t)stream);
+        if (e != cudaSuccess) return cuda_fail(e, "extrapolate launch");
+        return CB_OK;
+    }
+    size_t smem = 0;
+    rc = bulk_config(p, p->K, cb16, &A.stages, &smem);
     if (rc != CB_OK) return rc;
-    cudaError_t e = cbk::launch_extrapolate(A, p->K, cb16, grid, (cudaStream_t)stream);
+    A.wait_ns = p->wait_ns;
+    A.status = p->status_word();
+    A.withhold_first = p->withhold_first;
+    const int grid = (int)(tiles < p->dev.sms ? tiles : p->dev.sms);  // one CTA per SM
+    cudaError_t e = cbk::launch_extrapolate_bulk(A, p->K, cb16, grid, smem, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e, "extrapolate launch");
     return CB_OK;
 }
@@ -363,7 +402,9 @@ int cb_plan_create(const double* node_t, int n_nodes, int K, const cb_tensor_des
     }
 }
 
-size_t cb_plan_cache_bytes(const cb_plan* p) { return p ? p->slot_bytes * (size_t)p->K : 0; }
+size_t cb_plan_cache_bytes(const cb_plan* p) {
+    return p ? p->slot_bytes * (size_t)p->K + CB_STATUS_BYTES : 0;
+}
 
 int cb_plan_bind_cache(cb_plan* p, void* dev_ptr, size_t bytes) {
     if (!p || !dev_ptr || bytes < cb_plan_cache_bytes(p)) return CB_ERR_ARG;
@@ -371,6 +412,7 @@ int cb_plan_bind_cache(cb_plan* p, void* dev_ptr, size_t bytes) {
     p->cache = static_cast<unsigned char*>(dev_ptr);
     p->next = p->count = 0;
     p->has_last = false;
+    p->status_clear = false;  // zeroed on the stream of the first push
     return CB_OK;
 }
 
@@ -411,7 +453,13 @@ int cb_cache_push(cb_plan* p, const void* const* feats, cb_dtype feat_dtype, dou
     int grid = 0;
     rc = push_grid(p, sb, db, (int)tiles, &grid);
     if (rc != CB_OK) return rc;
-    cudaError_t e = cbk::launch_push(A, sb, db, grid, (cudaStream_t)stream);
+    cudaError_t e;
+    if (!p->status_clear) {
+        e = cudaMemsetAsync(p->status_word(), 0, sizeof(int), (cudaStream_t)stream);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
+        p->status_clear = true;
+    }
+    e = cbk::launch_push(A, sb, db, grid, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e, "push launch");
     // the pair (t, f_t) is now in H; the oldest entry was overwritten when full
     p->slot_t[p->next] = t;
@@ -489,6 +537,42 @@ int cb_plan_reset(cb_plan* p) {
     if (!p) return CB_ERR_ARG;
     p->next = p->count = 0;
     p->has_last = false;
+    return CB_OK;
+}
+
+int cb_plan_set_option(cb_plan* p, int option, int64_t value) {
+    if (!p) return CB_ERR_ARG;
+    switch (option) {
+    case CB_OPT_KERNEL:
+        if (value != CB_KERNEL_AUTO && value != CB_KERNEL_DIRECT && value != CB_KERNEL_BULK) return CB_ERR_ARG;
+        p->kernel = (int)value;
+        return CB_OK;
+    case CB_OPT_WAIT_NS:
+        if (value < 0) return CB_ERR_ARG;
+        p->wait_ns = (unsigned long long)value;
+        return CB_OK;
+    case CB_OPT_TEST_WITHHOLD:
+        if (value != 0 && value != 1) return CB_ERR_ARG;
+        p->withhold_first = (int)value;
+        return CB_OK;
+    default: return CB_ERR_ARG;
+    }
+}
+
+int cb_plan_device_status(cb_plan* p, int* status, void* stream) {
+    if (!p || !status) return CB_ERR_ARG;
+    if (!p->cache) return CB_ERR_UNBOUND;
+    if (!p->status_clear) {  // nothing has run since binding
+        *status = 0;
+        return CB_OK;
+    }
+    cudaStream_t s = (cudaStream_t)stream;
+    int v = 0;
+    cudaError_t e = cudaMemcpyAsync(&v, p->status_word(), sizeof(int), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(p->status_word(), 0, sizeof(int), s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(e, "device status");
+    *status = v;
     return CB_OK;
 }
 

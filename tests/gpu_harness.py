@@ -22,6 +22,7 @@ from paper_2608_23429_gb300 import workloads
 CB = {"bf16": cb.CB_BF16, "fp32": cb.CB_FP32}
 ORC = {"bf16": orc.BF16, "fp32": orc.FP32}
 TORCH = {"bf16": torch.bfloat16, "fp32": torch.float32}
+KERNEL = {"auto": cb.CB_KERNEL_AUTO, "direct": cb.CB_KERNEL_DIRECT, "bulk": cb.CB_KERNEL_BULK}
 FLOOR = 2.0 ** -40  # cancellation floor: |P| this small relative to sum|w F| is not resolvable
 
 
@@ -79,7 +80,7 @@ def merge(stats: list[dict]) -> dict:
 
 class Walk:
     def __init__(self, w: workloads.Workload, K: int | None = None, samples: int | None = None,
-                 seed: int = 0, device: str = "cuda", node_t=None):
+                 seed: int = 0, device: str = "cuda", node_t=None, kernel: str = "auto"):
         self.w = w
         self.K = K or w.K
         self.dev = torch.device(device)
@@ -92,6 +93,7 @@ class Walk:
         self.plan = cb.cb_plan_create(self.node_t, self.K, self.tensors, CB[self.cdt], w.t_min, w.t_max)
         self.cache = torch.empty(cb.cb_plan_cache_bytes(self.plan), dtype=torch.uint8, device=self.dev)
         cb.cb_plan_bind_cache(self.plan, self.cache, self.cache.numel())
+        cb.cb_plan_set_option(self.plan, cb.CB_OPT_KERNEL, KERNEL[kernel])
         self.H = orc.History(self.K)
         self.n_groups = cb.cb_plan_num_groups(self.plan)
         # sampled element indices: one set per element space (group or lone tensor)
@@ -139,6 +141,7 @@ class Walk:
             slot_t, head = ring
             cb.cb_extrapolate_ring(self.plan, slot_t, head, t, out_t, CB[out_dtype], resid, CB[resid_dtype])
         torch.cuda.synchronize()
+        assert cb.cb_plan_device_status(self.plan) == 0
         return out_t, resid, resid_host
 
     def _gidx(self, g):

@@ -95,12 +95,12 @@ def test_cache_layout_and_bind(cb):
     for dt, es in ((cb.CB_BF16, 2), (cb.CB_FP32, 4)):
         p = cb.cb_plan_create([3.0, 2.0, 1.0], 3, _tensors(numels), dt, 0.0, 3.0)
         slot = sum((n * es + 255) // 256 * 256 for n in numels)
-        assert cb.cb_plan_cache_bytes(p) == 3 * slot
+        assert cb.cb_plan_cache_bytes(p) == 3 * slot + cb.CB_STATUS_BYTES
         with pytest.raises(cb.CbError) as e:
-            cb.cb_plan_bind_cache(p, 0x1000 + 128, 3 * slot)
+            cb.cb_plan_bind_cache(p, 0x1000 + 128, 3 * slot + cb.CB_STATUS_BYTES)
         assert e.value.status == cb.CB_ERR_ALIGN
         with pytest.raises(cb.CbError) as e:
-            cb.cb_plan_bind_cache(p, 0x1000, 3 * slot - 1)
+            cb.cb_plan_bind_cache(p, 0x1000, 3 * slot + cb.CB_STATUS_BYTES - 1)
         assert e.value.status == cb.CB_ERR_ARG
         cb.cb_plan_destroy(p)
 
@@ -130,6 +130,14 @@ def test_validation_before_launch(cb):
     assert st("cb_weights", p, 850.0, w) == cb.CB_ERR_HISTORY_NOT_FULL
     slot_t, head, count = cb.cb_plan_history(p, 3)
     assert (head, count) == (0, 0)
+    # options
+    assert st("cb_plan_set_option", p, cb.CB_OPT_KERNEL, 7) == cb.CB_ERR_ARG
+    assert st("cb_plan_set_option", p, cb.CB_OPT_WAIT_NS, -1) == cb.CB_ERR_ARG
+    assert st("cb_plan_set_option", p, 99, 0) == cb.CB_ERR_ARG
+    for k in (cb.CB_KERNEL_DIRECT, cb.CB_KERNEL_BULK, cb.CB_KERNEL_AUTO):
+        cb.cb_plan_set_option(p, cb.CB_OPT_KERNEL, k)
+    # nothing has run since binding: the status read touches no device memory
+    assert cb.cb_plan_device_status(p) == 0
     assert cb.cb_plan_num_groups(p) == 1
     cb.cb_plan_destroy(p)
 

@@ -112,10 +112,10 @@ def test_tiny_fp32_polynomial_exact(cb, H):
 
 
 # ----------------------------------------- scaled schedules, every element
-@pytest.mark.parametrize("K", [3, 4])
-def test_dit256_scaled_full_schedule_fused(cb, H, K):
+@pytest.mark.parametrize("K,kernel", [(3, "bulk"), (4, "bulk"), (4, "direct")])
+def test_dit256_scaled_full_schedule_fused(cb, H, K, kernel):
     w = workloads.scaled(workloads.dit256(K), 8)
-    walk = H.Walk(w, K=K)
+    walk = H.Walk(w, K=K, kernel=kernel)
     mask, skipped = H.schedule_steps(w, K)
     agg_o, agg_r = [], []
     for s in range(w.T):
@@ -130,7 +130,7 @@ def test_dit256_scaled_full_schedule_fused(cb, H, K):
         agg_o.append(so)
         agg_r.append(sr)
     m = H.merge(agg_o)
-    print("dit256/8 K=%d outs" % K, m, "resid", H.merge(agg_r))
+    print("dit256/8 K=%d %s outs" % (K, kernel), m, "resid", H.merge(agg_r))
     # one-ulp differences arise where the exact sum of bf16 inputs with
     # near-dyadic weights lands on a bf16 rounding tie: the kernel breaks the
     # tie to even, the oracle by the ~1e-16 rounding noise of its fp64 weights
@@ -245,11 +245,12 @@ def test_ring_variant_and_rotation_bit_exact(cb, H):
 
 
 # ------------------------------------------------------------- edge cases
+@pytest.mark.parametrize("kernel", ["direct", "bulk"])
 @pytest.mark.parametrize("K,cache", [(1, "bf16"), (2, "fp32"), (5, "bf16"), (8, "bf16"), (8, "fp32")])
-def test_odd_sizes_every_element(cb, H, K, cache):
+def test_odd_sizes_every_element(cb, H, K, cache, kernel):
     w = _odd_workload(K, cache)
     nodes = [990.0 - 37.0 * k for k in range(K)]
-    walk = H.Walk(w, node_t=nodes)
+    walk = H.Walk(w, node_t=nodes, kernel=kernel)
     for k, t in enumerate(nodes):
         walk.push(t, k)
     t = nodes[-1] - 20.0
@@ -267,10 +268,11 @@ def test_odd_sizes_every_element(cb, H, K, cache):
     walk.close()
 
 
-def test_misaligned_outputs_take_scalar_path(cb, H):
+@pytest.mark.parametrize("kernel", ["direct", "bulk"])
+def test_misaligned_outputs_take_scalar_path(cb, H, kernel):
     w = _odd_workload(4)
     nodes = [950.0, 900.0, 850.0, 800.0]
-    walk = H.Walk(w, node_t=nodes)
+    walk = H.Walk(w, node_t=nodes, kernel=kernel)
     for k, t in enumerate(nodes):
         walk.push(t, k)
     t = 760.0
@@ -299,8 +301,9 @@ def test_target_on_node_returns_cached_features(cb, H):
     walk.close()
 
 
+@pytest.mark.parametrize("kernel", ["direct", "bulk"])
 @pytest.mark.parametrize("cache", ["bf16", "fp32"])
-def test_cancellation_stress(cb, H, cache):
+def test_cancellation_stress(cb, H, cache, kernel):
     """Histories whose extrapolation nearly cancels (|P| << sum |w F|), which
     sends elements through the compensated fallback of the fast path.
 
@@ -317,7 +320,7 @@ def test_cancellation_stress(cb, H, cache):
     tq = 0.43
     wt = orc.weights(nodes, tq, 0.0, 1.0)
     rng = np.random.default_rng(31)
-    walk = H.Walk(w, node_t=nodes)
+    walk = H.Walk(w, node_t=nodes, kernel=kernel)
     F = rng.standard_normal((2, K, n))
     if cache == "fp32":
         F = F.astype(np.float32).astype(np.float64)
@@ -414,4 +417,64 @@ def test_reset_and_history_errors(cb, H):
     assert cb.cb_plan_history(walk.plan, 2)[2] == 0
     with pytest.raises(cb.CbError):
         cb.cb_weights(walk.plan, 700.0, 2)
+    walk.close()
+
+
+# ------------------------------------------------- kernel variants, wait limit
+@pytest.mark.parametrize("name", ["flux", "dit256"])
+def test_direct_and_bulk_kernels_bit_identical(cb, H, name):
+    """Both skipped-step kernels run the same arithmetic: identical bits on a
+    full-size workload (outputs, and the fused hidden states on DiT-256)."""
+    w = workloads.flux() if name == "flux" else workloads.dit256(4)
+    walk = H.Walk(w)
+    mask, skipped = H.schedule_steps(w, w.K)
+    s_stop = skipped[len(skipped) // 2]
+    for s in range(s_stop):
+        if mask[s]:
+            walk.push(w.timesteps[s], s, )
+    t = w.timesteps[s_stop]
+    res = {}
+    for kern in ("direct", "bulk"):
+        cb.cb_plan_set_option(walk.plan, cb.CB_OPT_KERNEL, H.KERNEL[kern])
+        outs, resid, _ = walk.extrapolate(t, fused=(name == "dit256"), salt=5)
+        res[kern] = (outs, resid)
+    for a, b in zip(res["direct"][0], res["bulk"][0]):
+        assert torch.equal(a.view(torch.int16), b.view(torch.int16))
+    if name == "dit256":
+        for a, b in zip(res["direct"][1], res["bulk"][1]):
+            assert torch.equal(a.view(torch.int16), b.view(torch.int16))
+    walk.close()
+    torch.cuda.empty_cache()
+
+
+def test_bulk_wait_limit_reports_and_recovers(cb, H):
+    """The failure path of the bulk kernel's bounded waits, without a fault: the
+    producer announces every CTA's first unit but never issues its copies (a
+    flag that nothing sets), so the consumers' wait runs out after the limit.
+    The kernel must record it in the status word and return; the context stays
+    usable and the next launch is correct and clean."""
+    import time
+    w = workloads.scaled(workloads.pixart(), 16)
+    walk = H.Walk(w, kernel="bulk")
+    mask, skipped = H.schedule_steps(w, w.K)
+    for s in range(skipped[0]):
+        if mask[s]:
+            walk.push(w.timesteps[s], s)
+    t = w.timesteps[skipped[0]]
+    outs = [torch.empty(s.shape, dtype=torch.bfloat16, device="cuda") for s in w.tensors]
+    cb.cb_plan_set_option(walk.plan, cb.CB_OPT_WAIT_NS, 20_000_000)  # 20 ms
+    cb.cb_plan_set_option(walk.plan, cb.CB_OPT_TEST_WITHHOLD, 1)
+    t0 = time.perf_counter()
+    cb.cb_extrapolate(walk.plan, t, outs, cb.CB_BF16)
+    torch.cuda.synchronize()
+    elapsed = time.perf_counter() - t0
+    st = cb.cb_plan_device_status(walk.plan)
+    assert st & cb.CB_DEV_CONSUMER_TIMEOUT, st
+    assert st & cb.CB_DEV_PRODUCER_TIMEOUT, st
+    assert elapsed < 5.0
+    assert cb.cb_plan_device_status(walk.plan) == 0  # the read cleared it
+    cb.cb_plan_set_option(walk.plan, cb.CB_OPT_TEST_WITHHOLD, 0)
+    cb.cb_plan_set_option(walk.plan, cb.CB_OPT_WAIT_NS, 10 ** 9)
+    outs, _, _ = walk.extrapolate(t)
+    _assert_ok(walk.expected_and_compare(t, outs, None, None)[0], "after timeout")
     walk.close()
