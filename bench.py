@@ -278,11 +278,16 @@ def run_ours(args):
     outs = [torch.empty(t.shape, dtype=tdt, device=dev) for t in w.tensors]
     slot_elems = sum(t.numel for t in w.tensors)
     esz = 2 if w.cache_dtype == "bf16" else 4
-    bytes_step = slot_elems * esz * (K + 1)  # K slot reads + one output write
+    fused = w.fused if args.fused == "auto" else args.fused == "on"
+    n_groups = cb.cb_plan_num_groups(plan)
+    resid = [wl.hidden_state(w, g, dev) for g in range(n_groups)] if fused else None
+    resid_elems = sum(w.group_numel(g) for g in range(n_groups)) if fused else 0
+    # K slot reads + one output write (+ hidden state read and write)
+    bytes_step = slot_elems * esz * (K + 1) + resid_elems * 2 * 2
     t_targets = [w.timesteps[s] for s in targets]
 
     def step(k):
-        cb.cb_extrapolate(plan, t_targets[k % len(t_targets)], outs, cdt, stream=stream)
+        cb.cb_extrapolate(plan, t_targets[k % len(t_targets)], outs, cdt, resid, cb.CB_BF16, stream=stream)
 
     for k in range(args.warmup):
         step(k)
@@ -322,7 +327,7 @@ def run_ours(args):
     # predictions back; every copy is inside the timed region.
     e2e = None
     if not args.no_e2e:
-        e2e = run_e2e(args, torch, cb, wl, w, plan, cdt, tdt, dev, pushed, t_targets, bytes_step, ws)
+        e2e = run_e2e(args, torch, cb, wl, w, plan, cdt, tdt, dev, pushed, t_targets, bytes_step, ws, fused)
 
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu:
@@ -336,7 +341,8 @@ def run_ours(args):
     cb.cb_plan_destroy(plan)
     if rank == 0:
         desc = workload_description(w)
-        desc.update({"bytes_per_step": bytes_step, "targets": targets, "history_steps": pushed[-K:],
+        desc.update({"bytes_per_step": bytes_step, "fused_residual": fused, "targets": targets,
+                     "history_steps": pushed[-K:],
                      "l2": "inputs larger than L2 (no flush)", "launch": "1 grouped persistent kernel per step",
                      "parallelism": f"replicas x{ws}" if ws > 1 else "1 GPU"})
         line = {
@@ -358,29 +364,66 @@ def run_ours(args):
     return 0
 
 
-def run_e2e(args, torch, cb, wl, w, plan, cdt, tdt, dev, pushed, t_targets, bytes_step, ws):
+def host_memory_is_device_mapped(ptr: int) -> bool:
+    """True when a pinned host pointer is directly usable by kernels (UVA mapping)."""
+    import ctypes
+    try:
+        rt = ctypes.CDLL("libcudart.so.13")
+    except OSError:
+        return False
+    dptr = ctypes.c_void_p()
+    rc = rt.cudaHostGetDevicePointer(ctypes.byref(dptr), ctypes.c_void_p(ptr), 0)
+    return rc == 0 and dptr.value == ptr
+
+
+def run_e2e(args, torch, cb, wl, w, plan, cdt, tdt, dev, pushed, t_targets, bytes_step, ws, fused):
+    """One skipped step through the public API with every input and output in
+    pinned host memory: the K cached feature sets are pushed from the host, the
+    step is extrapolated, and the predictions (and hidden states) land in host
+    memory. zerocopy: the kernels read and write the pinned buffers over the
+    CPU-GPU link (they are device-mapped); copy: explicit staging copies."""
     K = w.K
     nodes = pushed[-K:]
     host_feats = []  # K sets of pinned host features (the full steps' outputs)
     for s in nodes:
         host_feats.append([wl.trajectory(w, i, w.timesteps[s], s, dev).cpu().pin_memory()
                            for i in range(len(w.tensors))])
-    dev_feats = [torch.empty(t.shape, dtype=tdt, device=dev) for t in w.tensors]
-    outs = [torch.empty(t.shape, dtype=tdt, device=dev) for t in w.tensors]
     host_outs = [torch.empty(t.shape, dtype=tdt).pin_memory() for t in w.tensors]
+    n_groups = cb.cb_plan_num_groups(plan)
+    host_resid = [wl.hidden_state(w, g, dev).cpu().pin_memory() for g in range(n_groups)] if fused else None
+    mode = args.e2e_mode
+    if mode == "zerocopy" and not host_memory_is_device_mapped(host_outs[0].data_ptr()):
+        mode = "copy"
     stream = torch.cuda.Stream(device=dev)
     slot = sum(t.numel for t in w.tensors) * (2 if w.cache_dtype == "bf16" else 4)
+    resid_bytes = sum(w.group_numel(g) for g in range(n_groups)) * 2 if fused else 0
+    if mode == "copy":
+        dev_feats = [torch.empty(t.shape, dtype=tdt, device=dev) for t in w.tensors]
+        outs = [torch.empty(t.shape, dtype=tdt, device=dev) for t in w.tensors]
+        resid = [torch.empty_like(r, device=dev) for r in host_resid] if fused else None
 
     def step(k):
         cb.cb_plan_reset(plan)
+        t = t_targets[k % len(t_targets)]
         with torch.cuda.stream(stream):
+            if mode == "zerocopy":
+                for j, s in enumerate(nodes):
+                    cb.cb_cache_push(plan, host_feats[j], cdt, w.timesteps[s], stream=stream)
+                cb.cb_extrapolate(plan, t, host_outs, cdt, host_resid, cb.CB_BF16, stream=stream)
+                return
             for j, s in enumerate(nodes):
                 for d, h in zip(dev_feats, host_feats[j]):
                     d.copy_(h, non_blocking=True)
                 cb.cb_cache_push(plan, dev_feats, cdt, w.timesteps[s], stream=stream)
-            cb.cb_extrapolate(plan, t_targets[k % len(t_targets)], outs, cdt, stream=stream)
+            if fused:
+                for d, h in zip(resid, host_resid):
+                    d.copy_(h, non_blocking=True)
+            cb.cb_extrapolate(plan, t, outs, cdt, resid, cb.CB_BF16, stream=stream)
             for h, o in zip(host_outs, outs):
                 h.copy_(o, non_blocking=True)
+            if fused:
+                for h, d in zip(host_resid, resid):
+                    h.copy_(d, non_blocking=True)
 
     steps = max(1, args.e2e_steps)
     for k in range(2):
@@ -394,8 +437,9 @@ def run_e2e(args, torch, cb, wl, w, plan, cdt, tdt, dev, pushed, t_targets, byte
     stream.synchronize()
     ms = max_over_ranks(a.elapsed_time(b) / steps, dev)
     return {"value": round(bytes_step * ws / (ms / 1e3) / 1e9, 2), "unit": "GB/s",
-            "h2d_bytes_per_step": K * slot, "d2h_bytes_per_step": slot, "ms_per_step": round(ms, 3),
-            "steps": steps}
+            "h2d_bytes_per_step": K * slot + resid_bytes, "d2h_bytes_per_step": slot + resid_bytes,
+            "ms_per_step": round(ms, 3), "steps": steps, "mode": mode,
+            "path": "cb_cache_push x K from host buffers + cb_extrapolate into host buffers"}
 
 
 def main():
@@ -405,6 +449,10 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--config", default="flux", choices=["dit256", "dit256-k3", "dit512", "pixart", "flux"])
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--fused", default="auto", choices=["auto", "on", "off"],
+                    help="add the predictions into the blocks' hidden states (auto: as the workload states)")
+    ap.add_argument("--e2e-mode", default="zerocopy", choices=["zerocopy", "copy"],
+                    help="e2e host buffers: read/written by the kernels over C2C, or staged by copies")
     ap.add_argument("--kernel", default="auto", choices=["auto", "direct", "bulk"],
                     help="skipped-step kernel variant (both compute identical bits)")
     ap.add_argument("--scale", type=int, default=1,

@@ -17,10 +17,13 @@
  *     and tau is the timestep mapped affinely onto [-1, 1] (Sec. 3.3).
  *
  * Conventions for every call:
- *   - Host/device: "device pointer" means memory of the current CUDA device;
- *     "host pointer" means ordinary process memory. The plan holds host state
- *     only; the caller owns and allocates every device buffer (cache arena,
- *     features, outputs, hidden states) and every stream.
+ *   - Host/device: "device pointer" means memory the current CUDA device's
+ *     kernels can address: its own memory, or host memory mapped into the
+ *     device's address space (pinned, UVA-mapped buffers, which the kernels
+ *     then read or write over the CPU-GPU link). "host pointer" means ordinary
+ *     process memory read by the host code. The plan holds host state only;
+ *     the caller owns and allocates every buffer (cache arena, features,
+ *     outputs, hidden states) and every stream.
  *   - Streams: `stream` is a cudaStream_t passed as void* (NULL = the legacy
  *     default stream). Device work is enqueued on it asynchronously; no call
  *     synchronises the device.
@@ -84,7 +87,8 @@ enum {
 /* Options of cb_plan_set_option. */
 enum {
     CB_OPT_KERNEL = 1,  /* skipped-step kernel: CB_KERNEL_AUTO (default), _DIRECT or _BULK */
-    CB_OPT_WAIT_NS = 2, /* limit of every device-side wait of the bulk kernel, ns (default 1e9) */
+    CB_OPT_WAIT_NS = 2, /* limit of every device-side wait of the bulk kernel, ns
+                           (default 1e9, at most 6e10) */
     CB_OPT_TEST_WITHHOLD = 3 /* 1: (tests of the failure path only) the bulk kernel's producer
                                 announces each CTA's first unit but never issues its copies, so
                                 that the consumers' wait runs out; outputs are then invalid */

@@ -36,6 +36,8 @@ struct ExtrapArgs {
     int resid_bf16;  // hidden states are bf16 (else fp32)
     int precise;     // 1: compensated (Dot2) arithmetic for every element
     int stages;                  // bulk variant: shared-memory pipeline depth
+    int stage_chunks;            // bulk variant: 8 KB chunks per stage (K, or K + 1 with hidden states)
+    int stage_x;                 // bulk variant: bf16 hidden states are staged as chunk K
     unsigned long long wait_ns;  // bulk variant: limit of every barrier wait
     int* status;                 // bulk variant: device status word (codes OR-ed in)
     int withhold_first;          // bulk variant, tests only: announce but never issue the first copies
@@ -67,7 +69,7 @@ cudaError_t launch_extrapolate(const ExtrapArgs& a, int K, bool cache_bf16, int 
 cudaError_t extrapolate_blocks_per_sm(int K, bool cache_bf16, int* blocks);
 
 // Bulk-copy pipeline variant (extrapolate_bulk.cu).
-size_t bulk_smem_bytes(int K, int stages);
+size_t bulk_smem_bytes(int chunks_per_stage, int stages);
 int bulk_threads();
 cudaError_t prepare_extrapolate_bulk(int K, bool cache_bf16, size_t smem);
 cudaError_t launch_extrapolate_bulk(const ExtrapArgs& a, int K, bool cache_bf16, int grid, size_t smem,

@@ -286,26 +286,33 @@ __device__ __forceinline__ void member_fast(const ExtrapArgs& A, long long moff,
 }
 
 // Fast path: hidden state <- bf16(x + sum_b s_b), guarded like the members.
-template <int K, bool CB16, int UV>
+// xload(u, x) supplies the 8 hidden-state values of vector u (global or shared
+// memory); exact(u, e, x_e, hi, lo) recomputes one guarded element with Dot2.
+template <int K, int UV, typename XLoad, typename Exact>
 __device__ __forceinline__ void resid_fast(const ExtrapArgs& A, int it, const long long (&ev)[UV],
-                                           const Acc<UV>& acc, void* resid) {
+                                           const Acc<UV>& acc, void* resid, XLoad xload, Exact exact) {
     const float g_res = (float)(K + A.nb[it] + 3) * kU * 1.01f;
 #pragma unroll
     for (int u = 0; u < UV; ++u) {
         float x[8], t[8];
         uint32_t pk[4];
-        load_x8(resid, true, ev[u], x);
+        xload(u, x);
 #pragma unroll
         for (int e = 0; e < 8; ++e) t[e] = acc.x[u][e] + x[e];
 #pragma unroll
         for (int i = 0; i < 4; ++i) pk[i] = pack_bf16x2(t[2 * i], t[2 * i + 1]);
+        unsigned bad = 0;
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-            if (!guard_ok(g_res, acc.y[u][e] + fabsf(x[e]), t[e])) {
-                float hi, lo;
-                exact_resid<CB16>(A, K, it, ev[u] + e, x[e], hi, lo);
-                set_half(pk, e, bf16_of_pair(hi, lo));
-            }
+        for (int e = 0; e < 8; ++e) bad |= guard_ok(g_res, acc.y[u][e] + fabsf(x[e]), t[e]) ? 0u : (1u << e);
+        while (bad) {
+            const int e = __ffs(bad) - 1;
+            bad &= bad - 1;
+            float xe = x[0];
+#pragma unroll
+            for (int i = 1; i < 8; ++i) xe = (e == i) ? x[i] : xe;
+            float hi, lo;
+            exact(u, e, xe, hi, lo);
+            set_half(pk, e, bf16_of_pair(hi, lo));
         }
         store_bf16x8(resid, ev[u], pk);
     }
@@ -354,13 +361,13 @@ __device__ __forceinline__ void member_precise(const ExtrapArgs& A, void* out, c
     }
 }
 
-template <int UV>
+template <int UV, typename XLoad>
 __device__ __forceinline__ void resid_precise(const ExtrapArgs& A, const long long (&ev)[UV], Acc<UV>& acc,
-                                              void* resid) {
+                                              void* resid, XLoad xload) {
 #pragma unroll
     for (int u = 0; u < UV; ++u) {
         float x[8], hi[8], lo[8];
-        load_x8(resid, A.resid_bf16, ev[u], x);
+        xload(u, x);
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
             float q;

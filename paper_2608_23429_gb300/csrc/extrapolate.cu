@@ -44,7 +44,8 @@ __device__ __forceinline__ void item_vectors(const ExtrapArgs& A, int it, const 
             load_member<K, CB16, UV>(A, A.m_off[first + m], ev, raw);
             member_precise<K, CB16, UV>(A, A.m_out[first + m], ev, raw, resid != nullptr, acc);
         }
-        if (resid) resid_precise<UV>(A, ev, acc, resid);
+        if (resid)
+            resid_precise<UV>(A, ev, acc, resid, [&](int u, float (&x)[8]) { load_x8(resid, A.resid_bf16, ev[u], x); });
     } else {
         Acc<UV> acc;
         acc.zero();
@@ -54,7 +55,12 @@ __device__ __forceinline__ void item_vectors(const ExtrapArgs& A, int it, const 
             member_fast<K, CB16, UV, false>(A, A.m_off[first + m], A.m_out[first + m], ev, raw, resid != nullptr,
                                             acc);
         }
-        if (resid) resid_fast<K, CB16, UV>(A, it, ev, acc, resid);
+        if (resid)
+            resid_fast<K, UV>(
+                A, it, ev, acc, resid, [&](int u, float (&x)[8]) { load_x8(resid, true, ev[u], x); },
+                [&](int u, int e, float xe, float& hi, float& lo) {
+                    exact_resid<CB16>(A, K, it, ev[u] + e, xe, hi, lo);
+                });
     }
 }
 

@@ -8,7 +8,12 @@
 // mbarrier (consumer warps). Eight consumer warps read their two 8-element
 // vectors of the K chunks from shared memory (the same element-to-thread map
 // as the direct kernel), release the stage, and compute and store from
-// registers. Nine warps leave each thread up to 168 registers. With S stages of K x 8 KB (S = 5 for K = 5) up to
+// registers. Nine warps leave each thread up to 168 registers. When hidden
+// states are updated, the producer also stages each tile's bf16 hidden state
+// (one more chunk with the group's last member) and the consumers hold the
+// group's member stages until the hidden state is written, so that the rare
+// guarded elements are recomputed from shared memory (the host guarantees
+// more stages than members, so holding cannot starve the producer). With S stages of K x 8 KB (S = 5 for K = 5) up to
 // ~160 KB per SM stay in flight independently of the consumers' register use,
 // which is what bounds the direct-load variant.
 //
@@ -28,6 +33,7 @@ constexpr int kBulkThreads = (kConsumerWarps + 1) * 32;
 constexpr int kChunkBytes = 8192;   // one history entry's share of a tile
 constexpr int kBarrierBytes = 256;  // full[S] and empty[S] barriers, S <= 16
 constexpr unsigned long long kMinDrainNs = 10000000ull;  // copies land in microseconds
+constexpr unsigned long long kMaxWaitNs = 60000000000ull;  // no wait outlives a minute
 
 __device__ __forceinline__ uint32_t smem_addr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
 
@@ -53,8 +59,10 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
     return ok != 0;
 }
 
-// Wait for the phase with the given parity to complete, for at most limit_ns.
+// Wait for the phase with the given parity to complete, for at most limit_ns
+// (never more than kMaxWaitNs).
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, unsigned long long limit_ns) {
+    if (limit_ns > kMaxWaitNs) limit_ns = kMaxWaitNs;
     if (mbar_try_wait(bar, parity)) return true;
     const unsigned long long t0 = now_ns();
     while (!mbar_try_wait(bar, parity))
@@ -106,6 +114,7 @@ __global__ void __launch_bounds__(kBulkThreads, 1) extrapolate_bulk_kernel(const
     }
     __syncthreads();
 
+    const int C = A.stage_chunks;
     if (warp == kConsumerWarps) {  // ---------------------------------- producer
         if (lane != 0) return;
         int it = 0;
@@ -121,21 +130,28 @@ __global__ void __launch_bounds__(kBulkThreads, 1) extrapolate_bulk_kernel(const
             const bool full_tile = A.vec_ok[it] && e0 + TE <= numel;
             const uint32_t bytes = full_tile ? (uint32_t)kChunkBytes : 0u;
             const int first = A.first[it];
-            for (int m = 0; m < A.nb[it]; ++m, ++u) {
+            const int nb = A.nb[it];
+            const unsigned char* resid = reinterpret_cast<const unsigned char*>(A.resid[it]);
+            for (int m = 0; m < nb; ++m, ++u) {
                 const uint32_t stage = u % (unsigned)S, q = u / (unsigned)S;
                 if (q > 0 && !mbar_wait(empty0 + 8u * stage, (q - 1) & 1u, A.wait_ns)) {
                     record(A.status, 2);
                     ok = false;
                     break;
                 }
-                mbar_expect_tx(full0 + 8u * stage, (uint32_t)K * bytes);
-                if (bytes && !(A.withhold_first && u == 0)) {
+                // the tile's bf16 hidden state travels with its last member
+                const bool with_x = A.stage_x && resid && full_tile && m == nb - 1;
+                const uint32_t xbytes = with_x ? (uint32_t)(TE * 2) : 0u;
+                mbar_expect_tx(full0 + 8u * stage, (uint32_t)K * bytes + xbytes);
+                if (A.withhold_first && u == 0) continue;
+                const uint32_t dst = buf0 + stage * (uint32_t)C * (uint32_t)kChunkBytes;
+                if (bytes) {
                     const unsigned char* src = A.cache + A.m_off[first + m] + e0 * ES;
 #pragma unroll
                     for (int j = 0; j < K; ++j)
-                        bulk_g2s(buf0 + (stage * K + j) * (uint32_t)kChunkBytes, src + A.slot_off[j], bytes,
-                                 full0 + 8u * stage);
+                        bulk_g2s(dst + j * (uint32_t)kChunkBytes, src + A.slot_off[j], bytes, full0 + 8u * stage);
                 }
+                if (xbytes) bulk_g2s(dst + K * (uint32_t)kChunkBytes, resid + e0 * 2, xbytes, full0 + 8u * stage);
             }
         }
         // never leave while copies into this CTA's shared memory are in flight
@@ -150,6 +166,8 @@ __global__ void __launch_bounds__(kBulkThreads, 1) extrapolate_bulk_kernel(const
 
     // ------------------------------------------------------------ consumers
     const int c = threadIdx.x;
+    const unsigned char* stages = smem + kBarrierBytes;
+    auto chunk = [&](uint32_t stage, int j) { return stages + ((size_t)stage * C + j) * kChunkBytes; };
     int it = 0;
     unsigned u = 0;
     for (int tile = blockIdx.x; tile < A.tiles_total; tile += gridDim.x) {
@@ -162,6 +180,10 @@ __global__ void __launch_bounds__(kBulkThreads, 1) extrapolate_bulk_kernel(const
         // whole aligned tiles come from shared memory; the ragged last tile of a
         // tensor and misaligned items take the compensated scalar path
         const bool full_tile = A.vec_ok[it] && e0 + TE <= numel;
+        // with a hidden state, every member's stage stays held until the hidden
+        // state is written, so that its guarded elements can be recomputed
+        const bool hold = full_tile && resid != nullptr;
+        const unsigned u0 = u;
         long long ev[U];
 #pragma unroll
         for (int v = 0; v < U; ++v) ev[v] = e0 + ((long long)v * kThreads + c) * kVecElems;
@@ -175,18 +197,19 @@ __global__ void __launch_bounds__(kBulkThreads, 1) extrapolate_bulk_kernel(const
             }
             RawVecs<K, CB16, U> raw;
             if (full_tile) {
-                const unsigned char* base = smem + kBarrierBytes + (size_t)stage * K * kChunkBytes;
 #pragma unroll
                 for (int v = 0; v < U; ++v)
 #pragma unroll
                     for (int j = 0; j < K; ++j) {
-                        const unsigned char* p = base + (size_t)j * kChunkBytes + (size_t)(ev[v] - e0) * ES;
+                        const unsigned char* p = chunk(stage, j) + (size_t)(ev[v] - e0) * ES;
                         raw[v][j][0] = *reinterpret_cast<const uint4*>(p);
                         if constexpr (!CB16) raw[v][j][CB16 ? 0 : 1] = *reinterpret_cast<const uint4*>(p + 16);
                     }
             }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(empty0 + 8u * stage);
+            if (!hold) {
+                __syncwarp();
+                if (lane == 0) mbar_arrive(empty0 + 8u * stage);
+            }
             if (full_tile) {
                 if (A.precise)
                     member_precise<K, CB16, U>(A, A.m_out[first + m], ev, raw, resid != nullptr, acc);
@@ -195,14 +218,43 @@ __global__ void __launch_bounds__(kBulkThreads, 1) extrapolate_bulk_kernel(const
                                                   resid != nullptr, acc);
             }
         }
-        if (full_tile) {
-            if (resid) {
-                if (A.precise)
-                    resid_precise<U>(A, ev, acc, resid);
+        if (hold) {
+            const uint32_t last = (u0 + nb - 1) % (unsigned)S;
+            auto xload = [&](int v, float (&x)[8]) {
+                if (A.stage_x)
+                    unpack_bf16x8(*reinterpret_cast<const uint4*>(chunk(last, K) + (size_t)(ev[v] - e0) * 2), x);
                 else
-                    resid_fast<K, CB16, U>(A, it, ev, acc, resid);
+                    load_x8(resid, A.resid_bf16, ev[v], x);
+            };
+            if (A.precise) {
+                resid_precise<U>(A, ev, acc, resid, xload);
+            } else {
+                // Dot2 of x + sum_b P_b for one element, from the held stages
+                auto exact = [&](int v, int e, float xe, float& hi, float& lo) {
+                    const size_t off = (size_t)(ev[v] - e0 + e) * ES;
+                    float tp = xe, tc = 0.0f;
+                    for (int m = 0; m < nb; ++m) {
+                        const uint32_t st = (u0 + m) % (unsigned)S;
+                        float p = 0.0f, cc = 0.0f, h, l, qq;
+#pragma unroll
+                        for (int j = 0; j < K; ++j) {
+                            const unsigned char* src = chunk(st, j) + off;
+                            const float f = CB16 ? __uint_as_float((uint32_t)(*reinterpret_cast<const uint16_t*>(src)) << 16)
+                                                 : *reinterpret_cast<const float*>(src);
+                            dot2_step(A.w_hi[j], A.w_lo[j], f, p, cc);
+                        }
+                        two_sum(p, cc, h, l);
+                        two_sum(tp, h, tp, qq);
+                        tc = __fadd_rn(tc, __fadd_rn(qq, l));
+                    }
+                    two_sum(tp, tc, hi, lo);
+                };
+                resid_fast<K, U>(A, it, ev, acc, resid, xload, exact);
             }
-        } else {
+            __syncwarp();
+            if (lane == 0)
+                for (int m = 0; m < nb; ++m) mbar_arrive(empty0 + 8u * ((u0 + m) % (unsigned)S));
+        } else if (!full_tile) {
             const long long end = e0 + TE < numel ? e0 + TE : numel;
             for (long long e = e0 + c; e < end; e += kThreads) scalar_element<CB16>(A, K, it, e);
         }
@@ -236,7 +288,9 @@ cudaError_t prepare_k(size_t smem) {
 
 }  // namespace
 
-size_t bulk_smem_bytes(int K, int stages) { return kBarrierBytes + (size_t)stages * K * kChunkBytes; }
+size_t bulk_smem_bytes(int chunks_per_stage, int stages) {
+    return kBarrierBytes + (size_t)stages * chunks_per_stage * kChunkBytes;
+}
 int bulk_threads() { return kBulkThreads; }
 
 cudaError_t prepare_extrapolate_bulk(int K, bool cache_bf16, size_t smem) {

@@ -64,7 +64,7 @@ struct DeviceInfo {
     int smem_optin = 0;                    // largest dynamic shared memory per CTA
     int occ_extrap[2][CB_MAX_K + 1] = {};  // [cache_bf16][K]
     int occ_push[2][2] = {};               // [src_bf16][dst_bf16]
-    int bulk_stages[2][CB_MAX_K + 1] = {};  // pipeline depth once the kernel is prepared
+    int bulk_stages[2][CB_MAX_K + 1] = {};  // 1 once the kernel's shared-memory limit is raised
 };
 
 }  // namespace
@@ -94,8 +94,9 @@ struct cb_plan {
     unsigned long long wait_ns = 1000000000ull;
     int withhold_first = 0;
     DeviceInfo dev;
-    std::unique_ptr<cbk::ExtrapArgs> eargs{new cbk::ExtrapArgs};
-    std::unique_ptr<cbk::PushArgs> pargs{new cbk::PushArgs};
+    // value-initialised: no field of a launch's arguments is ever left unset
+    std::unique_ptr<cbk::ExtrapArgs> eargs{new cbk::ExtrapArgs()};
+    std::unique_ptr<cbk::PushArgs> pargs{new cbk::PushArgs()};
 
     double tau(double t) const { return 2.0 * (t - t_min) / (t_max - t_min) - 1.0; }
     int* status_word() const { return reinterpret_cast<int*>(cache + slot_bytes * (size_t)K); }
@@ -134,21 +135,20 @@ int extrap_grid(cb_plan* p, int K, bool cb16, int tiles, int* grid) {
     return CB_OK;
 }
 
-// Pipeline depth of the bulk kernel: as many K x 8 KB stages as fit in one
-// CTA's shared memory (at most 8); the kernel's smem limit is raised once.
-int bulk_config(cb_plan* p, int K, bool cb16, int* stages, size_t* smem) {
-    int& st = p->dev.bulk_stages[cb16 ? 1 : 0][K];
-    if (st == 0) {
-        int s = 8;
-        while (s > 1 && cbk::bulk_smem_bytes(K, s) > (size_t)p->dev.smem_optin) --s;
-        if (cbk::bulk_smem_bytes(K, s) > (size_t)p->dev.smem_optin)
-            return cuda_fail(cudaErrorInvalidConfiguration, "bulk pipeline does not fit in shared memory");
-        cudaError_t e = cbk::prepare_extrapolate_bulk(K, cb16, cbk::bulk_smem_bytes(K, s));
+// Pipeline of the bulk kernel: as many stages of `chunks` 8 KB chunks as fit
+// in one CTA's shared memory (at most 8). The kernel's dynamic shared-memory
+// limit is raised to the device maximum once per instantiation.
+int bulk_config(cb_plan* p, int K, bool cb16, int chunks, int* stages, size_t* smem) {
+    int& prepared = p->dev.bulk_stages[cb16 ? 1 : 0][K];
+    if (prepared == 0) {
+        cudaError_t e = cbk::prepare_extrapolate_bulk(K, cb16, (size_t)p->dev.smem_optin);
         if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute");
-        st = s;
+        prepared = 1;
     }
-    *stages = st;
-    *smem = cbk::bulk_smem_bytes(K, st);
+    int s = 8;
+    while (s > 1 && cbk::bulk_smem_bytes(chunks, s) > (size_t)p->dev.smem_optin) --s;
+    *stages = cbk::bulk_smem_bytes(chunks, s) <= (size_t)p->dev.smem_optin ? s : 0;
+    *smem = cbk::bulk_smem_bytes(chunks, s);
     return CB_OK;
 }
 
@@ -293,6 +293,13 @@ int run_extrapolate(cb_plan* p, const Window& win, double t_target, void* const*
     A.precise = (any_out && out_dtype == CB_FP32) || (any_resid && resid_dtype == CB_FP32);
     if (items == 0) return CB_OK;  // nothing requested
 
+    A.wait_ns = p->wait_ns;
+    A.status = p->status_word();
+    A.withhold_first = p->withhold_first;
+    A.stages = 0;
+    A.stage_chunks = p->K;
+    A.stage_x = 0;
+
     rc = ensure_device(p);
     if (rc != CB_OK) return rc;
     if (p->kernel == CB_KERNEL_DIRECT) {
@@ -303,12 +310,24 @@ int run_extrapolate(cb_plan* p, const Window& win, double t_target, void* const*
         if (e != cudaSuccess) return cuda_fail(e, "extrapolate launch");
         return CB_OK;
     }
+    // bf16 hidden states travel through shared memory with the last member of
+    // their group; the pipeline must hold a whole group plus one stage ahead
+    int max_nb = 1;
+    for (int i = 0; i < items; ++i)
+        if (A.nb[i] > max_nb) max_nb = A.nb[i];
+    A.stage_x = any_resid && A.resid_bf16 ? 1 : 0;
+    A.stage_chunks = p->K + A.stage_x;
     size_t smem = 0;
-    rc = bulk_config(p, p->K, cb16, &A.stages, &smem);
+    rc = bulk_config(p, p->K, cb16, A.stage_chunks, &A.stages, &smem);
     if (rc != CB_OK) return rc;
-    A.wait_ns = p->wait_ns;
-    A.status = p->status_word();
-    A.withhold_first = p->withhold_first;
+    if (A.stages < max_nb + 1) {  // too deep for shared memory: the direct kernel instead
+        int grid = 0;
+        rc = extrap_grid(p, p->K, cb16, (int)tiles, &grid);
+        if (rc != CB_OK) return rc;
+        cudaError_t e = cbk::launch_extrapolate(A, p->K, cb16, grid, (cudaStream_t)stream);
+        if (e != cudaSuccess) return cuda_fail(e, "extrapolate launch");
+        return CB_OK;
+    }
     const int grid = (int)(tiles < p->dev.sms ? tiles : p->dev.sms);  // one CTA per SM
     cudaError_t e = cbk::launch_extrapolate_bulk(A, p->K, cb16, grid, smem, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e, "extrapolate launch");
@@ -548,7 +567,7 @@ int cb_plan_set_option(cb_plan* p, int option, int64_t value) {
         p->kernel = (int)value;
         return CB_OK;
     case CB_OPT_WAIT_NS:
-        if (value < 0) return CB_ERR_ARG;
+        if (value < 0 || value > 60000000000LL) return CB_ERR_ARG;
         p->wait_ns = (unsigned long long)value;
         return CB_OK;
     case CB_OPT_TEST_WITHHOLD:
