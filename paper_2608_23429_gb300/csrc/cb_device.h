@@ -70,7 +70,6 @@ cudaError_t extrapolate_blocks_per_sm(int K, bool cache_bf16, int* blocks);
 
 // Bulk-copy pipeline variant (extrapolate_bulk.cu).
 size_t bulk_smem_bytes(int chunks_per_stage, int stages);
-int bulk_threads();
 cudaError_t prepare_extrapolate_bulk(int K, bool cache_bf16, size_t smem);
 cudaError_t launch_extrapolate_bulk(const ExtrapArgs& a, int K, bool cache_bf16, int grid, size_t smem,
                                     cudaStream_t s);

@@ -1,21 +1,27 @@
 // Skipped-step kernel, bulk-copy pipeline variant (same arithmetic and bits as
 // extrapolate.cu; Sec. 3.3, Eq. for f_t; Alg. 1, extrapolation branch).
 //
-// One CTA per SM. A producer warp moves, for every work unit (one tile of one
+// One CTA per SM. A producer lane moves, for every work unit (one tile of one
 // branch tensor), the K history chunks of 8 KB each from HBM into a ring of
 // shared-memory stages with cp.async.bulk (the Blackwell bulk-copy engine),
 // each stage guarded by a "full" mbarrier (transaction bytes) and an "empty"
-// mbarrier (consumer warps). Eight consumer warps read their two 8-element
-// vectors of the K chunks from shared memory (the same element-to-thread map
-// as the direct kernel), release the stage, and compute and store from
-// registers. Nine warps leave each thread up to 168 registers. When hidden
-// states are updated, the producer also stages each tile's bf16 hidden state
-// (one more chunk with the group's last member) and the consumers hold the
-// group's member stages until the hidden state is written, so that the rare
-// guarded elements are recomputed from shared memory (the host guarantees
-// more stages than members, so holding cannot starve the producer). With S stages of K x 8 KB (S = 5 for K = 5) up to
-// ~160 KB per SM stay in flight independently of the consumers' register use,
+// mbarrier (one arrival per consumer warp). Consumer warps read their 8-element
+// vectors of the K chunks from shared memory, release the stage, and compute
+// and store from registers. With S stages of K x 8 KB (S = 5 for K = 5) up to
+// ~160 KB per SM stay in flight independently of the consumers' registers,
 // which is what bounds the direct-load variant.
+//
+// Two shapes, chosen per launch (GROUPED):
+//   * predictions only: 16 consumer warps with one vector each (17 warps, up
+//     to 96 registers per thread); more warps per scheduler hide the
+//     consumers' fixed latencies better (measured: +2 to +3 % of peak);
+//   * with hidden states: 8 consumer warps with two vectors each (the direct
+//     kernel's thread map, up to 168 registers). The producer also stages
+//     each tile's bf16 hidden state (one more chunk with the group's last
+//     member) and the consumers hold the group's member stages until the
+//     hidden state is written, so that the rare guarded elements are
+//     recomputed from shared memory (the host guarantees more stages than
+//     members, so holding cannot starve the producer).
 //
 // Every wait is bounded (%globaltimer). A wait that runs out records a code in
 // the plan's device status word and the thread returns; the producer then
@@ -28,8 +34,12 @@
 namespace cbk {
 namespace {
 
-constexpr int kConsumerWarps = 8;
-constexpr int kBulkThreads = (kConsumerWarps + 1) * 32;
+template <bool GROUPED>
+struct Shape {
+    static constexpr int consumer_warps = GROUPED ? 8 : 16;
+    static constexpr int consumers = consumer_warps * 32;
+    static constexpr int threads = consumers + 32;  // plus the producer warp
+};
 constexpr int kChunkBytes = 8192;   // one history entry's share of a tile
 constexpr int kBarrierBytes = 256;  // full[S] and empty[S] barriers, S <= 16
 constexpr unsigned long long kMinDrainNs = 10000000ull;  // copies land in microseconds
@@ -91,13 +101,20 @@ __device__ __forceinline__ void record(int* status, int code) {
     if (status) atomicOr(status, code);
 }
 
-template <int K, bool CB16>
-__global__ void __launch_bounds__(kBulkThreads, 1) extrapolate_bulk_kernel(const __grid_constant__ ExtrapArgs A) {
+// GROUPED: some item updates a hidden state (stage holding, hidden-state
+// staging, 8 consumer warps); prediction-only launches compile without that
+// bookkeeping and with 16 consumer warps.
+template <int K, bool CB16, bool GROUPED>
+__global__ void __launch_bounds__(Shape<GROUPED>::threads, 1)
+    extrapolate_bulk_kernel(const __grid_constant__ ExtrapArgs A) {
     extern __shared__ __align__(128) unsigned char smem[];
+    constexpr int NCW = Shape<GROUPED>::consumer_warps;
+    constexpr int NCT = Shape<GROUPED>::consumers;
     constexpr long long TE = tile_elems(CB16);  // 8 KB per history chunk for both cache types
     constexpr int ES = CB16 ? 2 : 4;
-    constexpr int U = vectors_per_thread(CB16);  // vectors per consumer thread per tile
-    static_assert(kConsumerWarps * 32 == kThreads, "consumers use the direct kernel's thread map");
+    constexpr int NV = (int)(TE / kVecElems);     // vectors per tile: 512 (bf16) or 256 (fp32)
+    constexpr int U = NV >= NCT ? NV / NCT : 1;   // vectors per consumer thread per tile
+    static_assert(NV % NCT == 0 || NCT % NV == 0, "vectors spread evenly over the consumers");
     static_assert(TE * ES == kChunkBytes, "one tile of one history entry is one chunk");
     const int S = A.stages;
     const uint32_t full0 = smem_addr(smem);
@@ -108,14 +125,14 @@ __global__ void __launch_bounds__(kBulkThreads, 1) extrapolate_bulk_kernel(const
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
             mbar_init(full0 + 8u * s, 1);
-            mbar_init(empty0 + 8u * s, kConsumerWarps);
+            mbar_init(empty0 + 8u * s, NCW);
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     __syncthreads();
 
-    const int C = A.stage_chunks;
-    if (warp == kConsumerWarps) {  // ---------------------------------- producer
+    const int C = GROUPED ? A.stage_chunks : K;
+    if (warp == NCW) {  // ---------------------------------- producer
         if (lane != 0) return;
         int it = 0;
         unsigned u = 0;
@@ -130,8 +147,8 @@ __global__ void __launch_bounds__(kBulkThreads, 1) extrapolate_bulk_kernel(const
             const bool full_tile = A.vec_ok[it] && e0 + TE <= numel;
             const uint32_t bytes = full_tile ? (uint32_t)kChunkBytes : 0u;
             const int first = A.first[it];
-            const int nb = A.nb[it];
-            const unsigned char* resid = reinterpret_cast<const unsigned char*>(A.resid[it]);
+            const int nb = GROUPED ? A.nb[it] : 1;
+            const unsigned char* resid = GROUPED ? reinterpret_cast<const unsigned char*>(A.resid[it]) : nullptr;
             for (int m = 0; m < nb; ++m, ++u) {
                 const uint32_t stage = u % (unsigned)S, q = u / (unsigned)S;
                 if (q > 0 && !mbar_wait(empty0 + 8u * stage, (q - 1) & 1u, A.wait_ns)) {
@@ -140,7 +157,7 @@ __global__ void __launch_bounds__(kBulkThreads, 1) extrapolate_bulk_kernel(const
                     break;
                 }
                 // the tile's bf16 hidden state travels with its last member
-                const bool with_x = A.stage_x && resid && full_tile && m == nb - 1;
+                const bool with_x = GROUPED && A.stage_x && resid && full_tile && m == nb - 1;
                 const uint32_t xbytes = with_x ? (uint32_t)(TE * 2) : 0u;
                 mbar_expect_tx(full0 + 8u * stage, (uint32_t)K * bytes + xbytes);
                 if (A.withhold_first && u == 0) continue;
@@ -174,19 +191,20 @@ __global__ void __launch_bounds__(kBulkThreads, 1) extrapolate_bulk_kernel(const
         while (tile >= A.tile_begin[it + 1]) ++it;
         const long long numel = A.numel[it];
         const long long e0 = (long long)(tile - A.tile_begin[it]) * TE;
-        const int nb = A.nb[it];
+        const int nb = GROUPED ? A.nb[it] : 1;
         const int first = A.first[it];
-        void* resid = A.resid[it];
+        void* resid = GROUPED ? A.resid[it] : nullptr;
         // whole aligned tiles come from shared memory; the ragged last tile of a
         // tensor and misaligned items take the compensated scalar path
         const bool full_tile = A.vec_ok[it] && e0 + TE <= numel;
         // with a hidden state, every member's stage stays held until the hidden
         // state is written, so that its guarded elements can be recomputed
-        const bool hold = full_tile && resid != nullptr;
+        const bool hold = GROUPED && full_tile && resid != nullptr;
+        const bool mine = NV >= NCT || c < NV;  // fp32 tiles have fewer vectors than consumers
         const unsigned u0 = u;
         long long ev[U];
 #pragma unroll
-        for (int v = 0; v < U; ++v) ev[v] = e0 + ((long long)v * kThreads + c) * kVecElems;
+        for (int v = 0; v < U; ++v) ev[v] = e0 + ((long long)v * NCT + c) * kVecElems;
         Acc<U> acc;
         acc.zero();
         for (int m = 0; m < nb; ++m, ++u) {
@@ -196,7 +214,7 @@ __global__ void __launch_bounds__(kBulkThreads, 1) extrapolate_bulk_kernel(const
                 return;
             }
             RawVecs<K, CB16, U> raw;
-            if (full_tile) {
+            if (full_tile && mine) {
 #pragma unroll
                 for (int v = 0; v < U; ++v)
 #pragma unroll
@@ -210,7 +228,7 @@ __global__ void __launch_bounds__(kBulkThreads, 1) extrapolate_bulk_kernel(const
                 __syncwarp();
                 if (lane == 0) mbar_arrive(empty0 + 8u * stage);
             }
-            if (full_tile) {
+            if (full_tile && mine) {
                 if (A.precise)
                     member_precise<K, CB16, U>(A, A.m_out[first + m], ev, raw, resid != nullptr, acc);
                 else
@@ -218,7 +236,7 @@ __global__ void __launch_bounds__(kBulkThreads, 1) extrapolate_bulk_kernel(const
                                                   resid != nullptr, acc);
             }
         }
-        if (hold) {
+        if (GROUPED && hold) {
             const uint32_t last = (u0 + nb - 1) % (unsigned)S;
             auto xload = [&](int v, float (&x)[8]) {
                 if (A.stage_x)
@@ -226,7 +244,8 @@ __global__ void __launch_bounds__(kBulkThreads, 1) extrapolate_bulk_kernel(const
                 else
                     load_x8(resid, A.resid_bf16, ev[v], x);
             };
-            if (A.precise) {
+            if (!mine) {
+            } else if (A.precise) {
                 resid_precise<U>(A, ev, acc, resid, xload);
             } else {
                 // Dot2 of x + sum_b P_b for one element, from the held stages
@@ -256,20 +275,26 @@ __global__ void __launch_bounds__(kBulkThreads, 1) extrapolate_bulk_kernel(const
                 for (int m = 0; m < nb; ++m) mbar_arrive(empty0 + 8u * ((u0 + m) % (unsigned)S));
         } else if (!full_tile) {
             const long long end = e0 + TE < numel ? e0 + TE : numel;
-            for (long long e = e0 + c; e < end; e += kThreads) scalar_element<CB16>(A, K, it, e);
+            for (long long e = e0 + c; e < end; e += NCT) scalar_element<CB16>(A, K, it, e);
         }
     }
 }
 
 template <int K, bool CB16>
-cudaError_t launch_k(const ExtrapArgs& a, int grid, size_t smem, cudaStream_t s) {
-    extrapolate_bulk_kernel<K, CB16><<<grid, kBulkThreads, smem, s>>>(a);
+cudaError_t launch_k(const ExtrapArgs& a, bool grouped, int grid, size_t smem, cudaStream_t s) {
+    if (grouped)
+        extrapolate_bulk_kernel<K, CB16, true><<<grid, Shape<true>::threads, smem, s>>>(a);
+    else
+        extrapolate_bulk_kernel<K, CB16, false><<<grid, Shape<false>::threads, smem, s>>>(a);
     return cudaGetLastError();
 }
 
 template <int K, bool CB16>
 cudaError_t prepare_k(size_t smem) {
-    return cudaFuncSetAttribute(extrapolate_bulk_kernel<K, CB16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(extrapolate_bulk_kernel<K, CB16, true>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    return cudaFuncSetAttribute(extrapolate_bulk_kernel<K, CB16, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)smem);
 }
 
@@ -291,7 +316,6 @@ cudaError_t prepare_k(size_t smem) {
 size_t bulk_smem_bytes(int chunks_per_stage, int stages) {
     return kBarrierBytes + (size_t)stages * chunks_per_stage * kChunkBytes;
 }
-int bulk_threads() { return kBulkThreads; }
 
 cudaError_t prepare_extrapolate_bulk(int K, bool cache_bf16, size_t smem) {
 #define P_BF(k) prepare_k<k, true>(smem)
@@ -306,8 +330,11 @@ cudaError_t prepare_extrapolate_bulk(int K, bool cache_bf16, size_t smem) {
 
 cudaError_t launch_extrapolate_bulk(const ExtrapArgs& a, int K, bool cache_bf16, int grid, size_t smem,
                                     cudaStream_t s) {
-#define L_BF(k) launch_k<k, true>(a, grid, smem, s)
-#define L_F32(k) launch_k<k, false>(a, grid, smem, s)
+    // fp32 caches have 256 vectors per tile: they keep the 8-consumer-warp shape
+    bool grouped = !cache_bf16;
+    for (int i = 0; i < a.n_items; ++i) grouped = grouped || a.resid[i] != nullptr || a.nb[i] > 1;
+#define L_BF(k) launch_k<k, true>(a, grouped, grid, smem, s)
+#define L_F32(k) launch_k<k, false>(a, grouped, grid, smem, s)
     if (cache_bf16) {
         CB_K_SWITCH(K, L_BF)
     }
