@@ -89,9 +89,14 @@ enum {
     CB_OPT_KERNEL = 1,  /* skipped-step kernel: CB_KERNEL_AUTO (default), _DIRECT or _BULK */
     CB_OPT_WAIT_NS = 2, /* limit of every device-side wait of the bulk kernel, ns
                            (default 1e9, at most 6e10) */
-    CB_OPT_TEST_WITHHOLD = 3 /* 1: (tests of the failure path only) the bulk kernel's producer
-                                announces each CTA's first unit but never issues its copies, so
-                                that the consumers' wait runs out; outputs are then invalid */
+    CB_OPT_TEST_WITHHOLD = 3, /* 1: (tests of the failure path only) the bulk kernel's producer
+                                 announces each CTA's first unit but never issues its copies, so
+                                 that the consumers' wait runs out; outputs are then invalid */
+    CB_OPT_PARTIAL_HISTORY = 4 /* 1: while H holds m < K entries (m >= 1), skipped steps use those m
+                                  (degree m-1 extrapolation; m = 1 reuses the newest features)
+                                  instead of failing with CB_ERR_HISTORY_NOT_FULL. This is Alg. 1
+                                  read literally ("retrieve cached features from H"); default 0,
+                                  the text's reading "provided |H| = n" */
 };
 enum { CB_KERNEL_AUTO = 0, CB_KERNEL_DIRECT = 1, CB_KERNEL_BULK = 2 };
 
@@ -177,9 +182,20 @@ int cb_extrapolate_ring(cb_plan* plan, const double* slot_t, int head, double t_
                         void* const* outs, cb_dtype out_dtype, void* const* resid,
                         cb_dtype resid_dtype, void* stream);
 
+/* Skipped step with caller-chosen weights: P_i = sum_j w_logical[j] F_{i,j}
+ * over the live history (the kernel of cb_extrapolate with the weights of
+ * Sec. 3.3's linear combination given directly, e.g. another node family's
+ * coefficients or finite-difference Taylor weights, see cb_taylor_weights).
+ * w_logical: host array of n doubles, oldest .. newest, n = K (or the number of
+ * live entries under CB_OPT_PARTIAL_HISTORY); outs, resid and errors as
+ * cb_extrapolate (non-finite weights: CB_ERR_ARG). */
+int cb_extrapolate_weights(cb_plan* plan, const double* w_logical, void* const* outs, cb_dtype out_dtype,
+                           void* const* resid, cb_dtype resid_dtype, void* stream);
+
 /* The fp64 weights cb_extrapolate would use for t_target on the live history
  * (Eq. barycentric_coeff), in logical order oldest .. newest. w_logical: host
- * array of K doubles. Errors: CB_ERR_ARG, CB_ERR_HISTORY_NOT_FULL. */
+ * array of n doubles, n = K (or the number of live entries under
+ * CB_OPT_PARTIAL_HISTORY). Errors: CB_ERR_ARG, CB_ERR_HISTORY_NOT_FULL. */
 int cb_weights(const cb_plan* plan, double t_target, double* w_logical);
 
 /* The "prepackaged" weight table (Sec. 3.3; Alg. 1, offline stage): for each
@@ -188,6 +204,17 @@ int cb_weights(const cb_plan* plan, double t_target, double* w_logical);
  * Errors: CB_ERR_ARG, CB_ERR_HISTORY_NOT_FULL (fewer than K nodes precede a
  * target). */
 int cb_plan_export_weights(const cb_plan* plan, const double* targets, int n_targets, double* table);
+
+/* Truncated-Taylor extrapolation weights (the Taylor expansion the paper
+ * compares against in Sec. 3.2, Fig. 4), with derivatives estimated by
+ * backward differences on n equispaced nodes: with h the node spacing and
+ * theta = (t_target - node_t[n-1]) / h,
+ *     f(t_target) ~ sum_{i<n} theta^i / i! * nabla^i f(node_t[n-1]),
+ *     nabla^i f_n = sum_{k<=i} (-1)^k C(i, k) f_{n-k}.
+ * w: host array of n doubles (oldest .. newest) for cb_extrapolate_weights.
+ * n = 1 gives w = (1): reuse of the newest features. Errors: CB_ERR_ARG (n out
+ * of [1, CB_MAX_K], nodes not equispaced), CB_ERR_NODES_DEGENERATE. */
+int cb_taylor_weights(const double* node_t, int n, double t_target, double* w);
 
 /* Introspection of H: slot_t (host, K doubles) receives each slot's time,
  * head the slot of the oldest entry, count the number of entries (<= K).

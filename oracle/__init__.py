@@ -52,6 +52,7 @@ def lib():
         L.orc_rho.argtypes, L.orc_rho.restype = [P, I, P], I
         L.orc_bary_coeff.argtypes, L.orc_bary_coeff.restype = [P, P, I, D, P], I
         L.orc_lagrange_basis.argtypes, L.orc_lagrange_basis.restype = [P, I, D, P], I
+        L.orc_taylor_weights.argtypes, L.orc_taylor_weights.restype = [P, I, D, P], I
         L.orc_convert.argtypes, L.orc_convert.restype = [P, I, I64, P, I], None
         L.orc_extrapolate.argtypes = [I, I, P, I, P, P, I, I64, P, I, P, I, I]
         L.orc_extrapolate.restype = I
@@ -133,6 +134,15 @@ def lagrange_basis(x, xq: float) -> np.ndarray:
     out = np.empty_like(x)
     if lib().orc_lagrange_basis(_ptr(x), x.size, float(xq), _ptr(out)) != 0:
         raise ValueError("duplicate nodes")
+    return out
+
+
+def taylor_weights(x, xq: float) -> np.ndarray:
+    """Truncated-Taylor weights with backward-difference derivatives (equispaced x)."""
+    x = _f64(x)
+    out = np.empty_like(x)
+    if lib().orc_taylor_weights(_ptr(x), x.size, float(xq), _ptr(out)) != 0:
+        raise ValueError("degenerate nodes")
     return out
 
 

@@ -19,6 +19,10 @@
  *   orc_bary_coeff      Sec. 3.2, Eq. barycentric_coeff:
  *                       w_j = (rho_j / (x - x_j)) / sum_i rho_i / (x - x_i).
  *   orc_lagrange_basis  App. A: l_j(x) = prod_{k != j} (x - x_k) / (x_j - x_k).
+ *   orc_taylor_weights  Sec. 3.2, Fig. 4's Taylor expansion: f(t) ~ sum_i theta^i/i!
+ *                       times the i-th backward difference at the newest node
+ *                       (derivatives estimated on equispaced nodes), written as
+ *                       one weight per node.
  *   orc_extrapolate     Sec. 3.3 Eq. for f_t (Alg. 1, extrapolation branch):
  *                       f_t = sum_j w_j f_{s_j}, per element, in fp64, then one
  *                       rounding to the output type; optionally the block
@@ -159,6 +163,32 @@ int orc_lagrange_basis(const double* x, int n, double xq, double* l) {
             p *= (xq - x[k]) / (x[j] - x[k]);
         }
         l[j] = p;
+    }
+    return 0;
+}
+
+/* Weight of node j (0 = oldest) in the truncated Taylor series about the
+ * newest node: each backward difference nabla^i f_n = sum_k (-1)^k C(i,k)
+ * f_{n-k} is spread over the nodes it touches. Plain nested loops; C(i,k) and
+ * i! from their products. */
+int orc_taylor_weights(const double* x, int n, double xq, double* w) {
+    if (n < 1) return -1;
+    double h = n >= 2 ? x[n - 1] - x[n - 2] : 1.0;
+    if (n >= 2 && h == 0.0) return -1;
+    double theta = n >= 2 ? (xq - x[n - 1]) / h : 0.0;
+    for (int j = 0; j < n; ++j) w[j] = 0.0;
+    for (int i = 0; i < n; ++i) {
+        double fact = 1.0, pw = 1.0;
+        for (int q = 1; q <= i; ++q) {
+            fact *= q;
+            pw *= theta;
+        }
+        for (int k = 0; k <= i; ++k) {
+            double c = 1.0; /* C(i, k) = i! / (k! (i-k)!) */
+            for (int q = 1; q <= k; ++q) c = c * (i - k + q) / q;
+            double sign = (k % 2 == 0) ? 1.0 : -1.0;
+            w[n - 1 - k] += pw / fact * sign * c;
+        }
     }
     return 0;
 }

@@ -25,7 +25,7 @@ _lib = ctypes.CDLL(LIB_PATH)
 
 CB_BF16, CB_FP32 = 0, 1
 CB_MAX_K, CB_MAX_TENSORS, CB_MAX_BRANCHES, CB_CACHE_ALIGN, CB_STATUS_BYTES = 8, 256, 4, 256, 256
-CB_OPT_KERNEL, CB_OPT_WAIT_NS, CB_OPT_TEST_WITHHOLD = 1, 2, 3
+CB_OPT_KERNEL, CB_OPT_WAIT_NS, CB_OPT_TEST_WITHHOLD, CB_OPT_PARTIAL_HISTORY = 1, 2, 3, 4
 CB_KERNEL_AUTO, CB_KERNEL_DIRECT, CB_KERNEL_BULK = 0, 1, 2
 CB_DEV_CONSUMER_TIMEOUT, CB_DEV_PRODUCER_TIMEOUT, CB_DEV_DRAIN_TIMEOUT = 1, 2, 4
 CB_OK, CB_ERR_ARG, CB_ERR_ALIGN, CB_ERR_NODES_DEGENERATE = 0, -1, -2, -3
@@ -47,7 +47,9 @@ _sig = {
     "cb_cache_push": ([_P, _PP, _I, _D, _P], _I),
     "cb_extrapolate": ([_P, _D, _PP, _I, _PP, _I, _P], _I),
     "cb_extrapolate_ring": ([_P, _P, _I, _D, _PP, _I, _PP, _I, _P], _I),
+    "cb_extrapolate_weights": ([_P, _P, _PP, _I, _PP, _I, _P], _I),
     "cb_weights": ([_P, _D, _P], _I),
+    "cb_taylor_weights": ([_P, _I, _D, _P], _I),
     "cb_plan_export_weights": ([_P, _P, _I, _P], _I),
     "cb_plan_history": ([_P, _P, _P, _P], _I),
     "cb_plan_reset": ([_P], _I),
@@ -151,9 +153,25 @@ def cb_extrapolate_ring(plan, slot_t, head: int, t_target: float, outs, out_dtyp
            "cb_extrapolate_ring")
 
 
-def cb_weights(plan, t_target: float, K: int) -> np.ndarray:
-    w = np.empty(K, dtype=np.float64)
+def cb_extrapolate_weights(plan, w_logical, outs, out_dtype: int, resid=None, resid_dtype: int = CB_BF16,
+                           stream=None) -> None:
+    w = _f64(w_logical)
+    _check(_lib.cb_extrapolate_weights(plan, w.ctypes.data, _ptr_array(outs), out_dtype, _ptr_array(resid),
+                                       resid_dtype, _stream(stream)), "cb_extrapolate_weights")
+
+
+def cb_weights(plan, t_target: float, n: int) -> np.ndarray:
+    """Weights over the n live history entries (n = K, or fewer under partial history)."""
+    w = np.empty(n, dtype=np.float64)
     _check(_lib.cb_weights(plan, float(t_target), w.ctypes.data), "cb_weights")
+    return w
+
+
+def cb_taylor_weights(node_t, t_target: float) -> np.ndarray:
+    node_t = _f64(node_t)
+    w = np.empty(node_t.size, dtype=np.float64)
+    _check(_lib.cb_taylor_weights(node_t.ctypes.data, node_t.size, float(t_target), w.ctypes.data),
+           "cb_taylor_weights")
     return w
 
 

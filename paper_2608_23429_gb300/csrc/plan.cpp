@@ -93,6 +93,7 @@ struct cb_plan {
     int kernel = CB_KERNEL_AUTO;
     unsigned long long wait_ns = 1000000000ull;
     int withhold_first = 0;
+    bool partial = false;  // extrapolate from fewer than K entries while H fills
     DeviceInfo dev;
     // value-initialised: no field of a launch's arguments is ever left unset
     std::unique_ptr<cbk::ExtrapArgs> eargs{new cbk::ExtrapArgs()};
@@ -168,8 +169,9 @@ int push_grid(cb_plan* p, bool sb, bool db, int tiles, int* grid) {
 
 bool aligned(const void* ptr, size_t a) { return ((uintptr_t)ptr % a) == 0; }
 
-// Logical history times (oldest first) and the slot of each entry.
+// Logical history window: n entries, oldest first, with the slot of each.
 struct Window {
+    int n;
     double t[CB_MAX_K];
     double tau[CB_MAX_K];
     int slot[CB_MAX_K];
@@ -180,35 +182,46 @@ struct Window {
 bool window_rho(const cb_plan* p, const Window& w, double* rho) {
     const int K = p->K;
     const int n = (int)p->node_t.size();
-    for (int i = 0; i + K <= n; ++i) {
-        if (p->node_t[i] != w.t[0]) continue;
-        bool match = true;
-        for (int j = 1; j < K && match; ++j) match = p->node_t[i + j] == w.t[j];
-        if (match) {
-            std::memcpy(rho, &p->rho_win[(size_t)i * K], sizeof(double) * K);
-            return true;
+    if (w.n == K) {
+        for (int i = 0; i + K <= n; ++i) {
+            if (p->node_t[i] != w.t[0]) continue;
+            bool match = true;
+            for (int j = 1; j < K && match; ++j) match = p->node_t[i + j] == w.t[j];
+            if (match) {
+                std::memcpy(rho, &p->rho_win[(size_t)i * K], sizeof(double) * K);
+                return true;
+            }
         }
     }
-    return rho_of(w.tau, K, rho);
+    return rho_of(w.tau, w.n, rho);
 }
 
 int weights_for(const cb_plan* p, const Window& w, double t_target, double* out) {
     if (!std::isfinite(t_target)) return CB_ERR_ARG;
     double rho[CB_MAX_K];
     if (!window_rho(p, w, rho)) return CB_ERR_NODES_DEGENERATE;
-    for (int j = 0; j < p->K; ++j)
+    for (int j = 0; j < w.n; ++j)
         if (t_target == w.t[j]) {  // the target is a cached node: return it exactly
-            for (int i = 0; i < p->K; ++i) out[i] = (i == j) ? 1.0 : 0.0;
+            for (int i = 0; i < w.n; ++i) out[i] = (i == j) ? 1.0 : 0.0;
             return CB_OK;
         }
-    coeff_of(w.tau, rho, p->K, p->tau(t_target), out);
+    coeff_of(w.tau, rho, w.n, p->tau(t_target), out);
     return CB_OK;
 }
 
-Window live_window(const cb_plan* p) {
+// Entries a skipped step may use: all K once H is full; with partial history
+// enabled, whatever H holds (at least one); otherwise none.
+int live_entries(const cb_plan* p) {
+    if (p->count == p->K) return p->K;
+    if (p->partial && p->count >= 1) return p->count;
+    return 0;
+}
+
+Window live_window(const cb_plan* p, int n) {
     Window w{};
+    w.n = n;
     const int o = p->oldest();
-    for (int j = 0; j < p->K; ++j) {
+    for (int j = 0; j < n; ++j) {
         w.slot[j] = (o + j) % p->K;
         w.t[j] = p->slot_t[w.slot[j]];
         w.tau[j] = p->tau(w.t[j]);
@@ -216,10 +229,12 @@ Window live_window(const cb_plan* p) {
     return w;
 }
 
-int run_extrapolate(cb_plan* p, const Window& win, double t_target, void* const* outs, cb_dtype out_dtype,
-                    void* const* resid, cb_dtype resid_dtype, void* stream) {
+// One skipped-step launch over the window `win` with the fp64 weights w[0..n).
+int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs, cb_dtype out_dtype,
+               void* const* resid, cb_dtype resid_dtype, void* stream) {
     if (!p->cache) return CB_ERR_UNBOUND;
-    if (p->count < p->K) return CB_ERR_HISTORY_NOT_FULL;
+    const int K = win.n;
+    if (K < 1 || p->count < K) return CB_ERR_HISTORY_NOT_FULL;
     if (!valid_dtype(out_dtype) || !valid_dtype(resid_dtype)) return CB_ERR_ARG;
     const int n = (int)p->tensors.size();
     const int ng = (int)p->groups.size();
@@ -231,16 +246,16 @@ int run_extrapolate(cb_plan* p, const Window& win, double t_target, void* const*
         for (int g = 0; g < ng; ++g)
             if (resid[g] && !aligned(resid[g], res)) return CB_ERR_ALIGN;
 
-    double w[CB_MAX_K];
-    int rc = weights_for(p, win, t_target, w);
-    if (rc != CB_OK) return rc;
+    for (int j = 0; j < K; ++j)
+        if (!std::isfinite(w[j])) return CB_ERR_ARG;
+    int rc = CB_OK;
 
     cbk::ExtrapArgs& A = *p->eargs;
     const bool cb16 = p->cache_dtype == CB_BF16;
     const long long te = cbk::tile_elems(cb16);
     A.cache = p->cache;
     for (int j = 0; j < CB_MAX_K; ++j) {
-        const bool on = j < p->K;
+        const bool on = j < K;
         A.slot_off[j] = on ? (long long)win.slot[j] * (long long)p->slot_bytes : 0;
         const float hi = on ? (float)w[j] : 0.0f;
         A.w_hi[j] = hi;
@@ -297,16 +312,16 @@ int run_extrapolate(cb_plan* p, const Window& win, double t_target, void* const*
     A.status = p->status_word();
     A.withhold_first = p->withhold_first;
     A.stages = 0;
-    A.stage_chunks = p->K;
+    A.stage_chunks = K;
     A.stage_x = 0;
 
     rc = ensure_device(p);
     if (rc != CB_OK) return rc;
     if (p->kernel == CB_KERNEL_DIRECT) {
         int grid = 0;
-        rc = extrap_grid(p, p->K, cb16, (int)tiles, &grid);
+        rc = extrap_grid(p, K, cb16, (int)tiles, &grid);
         if (rc != CB_OK) return rc;
-        cudaError_t e = cbk::launch_extrapolate(A, p->K, cb16, grid, (cudaStream_t)stream);
+        cudaError_t e = cbk::launch_extrapolate(A, K, cb16, grid, (cudaStream_t)stream);
         if (e != cudaSuccess) return cuda_fail(e, "extrapolate launch");
         return CB_OK;
     }
@@ -316,20 +331,20 @@ int run_extrapolate(cb_plan* p, const Window& win, double t_target, void* const*
     for (int i = 0; i < items; ++i)
         if (A.nb[i] > max_nb) max_nb = A.nb[i];
     A.stage_x = any_resid && A.resid_bf16 ? 1 : 0;
-    A.stage_chunks = p->K + A.stage_x;
+    A.stage_chunks = K + A.stage_x;
     size_t smem = 0;
-    rc = bulk_config(p, p->K, cb16, A.stage_chunks, &A.stages, &smem);
+    rc = bulk_config(p, K, cb16, A.stage_chunks, &A.stages, &smem);
     if (rc != CB_OK) return rc;
     if (A.stages < max_nb + 1) {  // too deep for shared memory: the direct kernel instead
         int grid = 0;
-        rc = extrap_grid(p, p->K, cb16, (int)tiles, &grid);
+        rc = extrap_grid(p, K, cb16, (int)tiles, &grid);
         if (rc != CB_OK) return rc;
-        cudaError_t e = cbk::launch_extrapolate(A, p->K, cb16, grid, (cudaStream_t)stream);
+        cudaError_t e = cbk::launch_extrapolate(A, K, cb16, grid, (cudaStream_t)stream);
         if (e != cudaSuccess) return cuda_fail(e, "extrapolate launch");
         return CB_OK;
     }
     const int grid = (int)(tiles < p->dev.sms ? tiles : p->dev.sms);  // one CTA per SM
-    cudaError_t e = cbk::launch_extrapolate_bulk(A, p->K, cb16, grid, smem, (cudaStream_t)stream);
+    cudaError_t e = cbk::launch_extrapolate_bulk(A, K, cb16, grid, smem, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e, "extrapolate launch");
     return CB_OK;
 }
@@ -492,30 +507,74 @@ int cb_cache_push(cb_plan* p, const void* const* feats, cb_dtype feat_dtype, dou
 int cb_extrapolate(cb_plan* p, double t_target, void* const* outs, cb_dtype out_dtype, void* const* resid,
                    cb_dtype resid_dtype, void* stream) {
     if (!p) return CB_ERR_ARG;
-    if (p->count < p->K) return p->cache ? CB_ERR_HISTORY_NOT_FULL : CB_ERR_UNBOUND;
-    return run_extrapolate(p, live_window(p), t_target, outs, out_dtype, resid, resid_dtype, stream);
+    const int n = live_entries(p);
+    if (n == 0) return p->cache ? CB_ERR_HISTORY_NOT_FULL : CB_ERR_UNBOUND;
+    const Window win = live_window(p, n);
+    double w[CB_MAX_K];
+    const int rc = weights_for(p, win, t_target, w);
+    if (rc != CB_OK) return rc;
+    return run_launch(p, win, w, outs, out_dtype, resid, resid_dtype, stream);
 }
 
 int cb_extrapolate_ring(cb_plan* p, const double* slot_t, int head, double t_target, void* const* outs,
                         cb_dtype out_dtype, void* const* resid, cb_dtype resid_dtype, void* stream) {
     if (!p || !slot_t || head < 0 || head >= (p ? p->K : 1)) return CB_ERR_ARG;
     if (p->count < p->K) return p->cache ? CB_ERR_HISTORY_NOT_FULL : CB_ERR_UNBOUND;
-    Window w{};
+    Window win{};
+    win.n = p->K;
     for (int j = 0; j < p->K; ++j) {
-        w.slot[j] = (head + j) % p->K;
-        w.t[j] = slot_t[w.slot[j]];
-        if (!std::isfinite(w.t[j])) return CB_ERR_ARG;
-        w.tau[j] = p->tau(w.t[j]);
+        win.slot[j] = (head + j) % p->K;
+        win.t[j] = slot_t[win.slot[j]];
+        if (!std::isfinite(win.t[j])) return CB_ERR_ARG;
+        win.tau[j] = p->tau(win.t[j]);
         for (int i = 0; i < j; ++i)
-            if (w.t[i] == w.t[j]) return CB_ERR_NODES_DEGENERATE;
+            if (win.t[i] == win.t[j]) return CB_ERR_NODES_DEGENERATE;
     }
-    return run_extrapolate(p, w, t_target, outs, out_dtype, resid, resid_dtype, stream);
+    double w[CB_MAX_K];
+    const int rc = weights_for(p, win, t_target, w);
+    if (rc != CB_OK) return rc;
+    return run_launch(p, win, w, outs, out_dtype, resid, resid_dtype, stream);
+}
+
+int cb_extrapolate_weights(cb_plan* p, const double* w_logical, void* const* outs, cb_dtype out_dtype,
+                           void* const* resid, cb_dtype resid_dtype, void* stream) {
+    if (!p || !w_logical) return CB_ERR_ARG;
+    const int n = live_entries(p);
+    if (n == 0) return p->cache ? CB_ERR_HISTORY_NOT_FULL : CB_ERR_UNBOUND;
+    return run_launch(p, live_window(p, n), w_logical, outs, out_dtype, resid, resid_dtype, stream);
 }
 
 int cb_weights(const cb_plan* p, double t_target, double* w_logical) {
     if (!p || !w_logical) return CB_ERR_ARG;
-    if (p->count < p->K) return CB_ERR_HISTORY_NOT_FULL;
-    return weights_for(p, live_window(p), t_target, w_logical);
+    const int n = live_entries(p);
+    if (n == 0) return CB_ERR_HISTORY_NOT_FULL;
+    return weights_for(p, live_window(p, n), t_target, w_logical);
+}
+
+int cb_taylor_weights(const double* node_t, int n, double t_target, double* w) {
+    if (!node_t || !w || n < 1 || n > CB_MAX_K || !std::isfinite(t_target)) return CB_ERR_ARG;
+    for (int i = 0; i < n; ++i)
+        if (!std::isfinite(node_t[i])) return CB_ERR_ARG;
+    double h = 1.0;
+    if (n >= 2) {
+        h = node_t[n - 1] - node_t[n - 2];
+        if (h == 0.0) return CB_ERR_NODES_DEGENERATE;
+        for (int i = 1; i < n; ++i)  // equispaced nodes only
+            if (std::fabs((node_t[i] - node_t[i - 1]) - h) > 1e-9 * std::fabs(h)) return CB_ERR_ARG;
+    }
+    const double theta = n >= 2 ? (t_target - node_t[n - 1]) / h : 0.0;
+    // f(t) ~ sum_i theta^i / i! nabla^i f_n, nabla^i f_n = sum_k (-1)^k C(i, k) f_{n-k}
+    for (int j = 0; j < n; ++j) w[j] = 0.0;
+    double pow_fact = 1.0;  // theta^i / i!
+    for (int i = 0; i < n; ++i) {
+        if (i > 0) pow_fact *= theta / i;
+        double binom = 1.0;  // C(i, k)
+        for (int k = 0; k <= i; ++k) {
+            if (k > 0) binom = binom * (i - k + 1) / k;
+            w[n - 1 - k] += pow_fact * ((k & 1) ? -binom : binom);
+        }
+    }
+    return CB_OK;
 }
 
 int cb_plan_export_weights(const cb_plan* p, const double* targets, int n_targets, double* table) {
@@ -533,6 +592,7 @@ int cb_plan_export_weights(const cb_plan* p, const double* targets, int n_target
         }
         if (last + 1 < K) return CB_ERR_HISTORY_NOT_FULL;
         Window w{};
+        w.n = K;
         for (int j = 0; j < K; ++j) {
             w.t[j] = p->node_t[last - K + 1 + j];
             w.tau[j] = p->node_tau[last - K + 1 + j];
@@ -569,6 +629,10 @@ int cb_plan_set_option(cb_plan* p, int option, int64_t value) {
     case CB_OPT_WAIT_NS:
         if (value < 0 || value > 60000000000LL) return CB_ERR_ARG;
         p->wait_ns = (unsigned long long)value;
+        return CB_OK;
+    case CB_OPT_PARTIAL_HISTORY:
+        if (value != 0 && value != 1) return CB_ERR_ARG;
+        p->partial = value != 0;
         return CB_OK;
     case CB_OPT_TEST_WITHHOLD:
         if (value != 0 && value != 1) return CB_ERR_ARG;

@@ -126,7 +126,7 @@ class Walk:
 
     # ---- skipped step
     def extrapolate(self, t: float, out_dtype: str = "bf16", fused: bool = False, outs: bool = True,
-                    resid_dtype: str = "bf16", ring=None, salt: int = 0):
+                    resid_dtype: str = "bf16", ring=None, salt: int = 0, explicit=None):
         w = self.w
         out_t = [torch.empty(s.shape, dtype=TORCH[out_dtype], device=self.dev) for s in w.tensors] if outs else None
         resid = None
@@ -135,7 +135,9 @@ class Walk:
             resid = [workloads.hidden_state(w, g, self.dev, TORCH[resid_dtype], salt=salt)
                      for g in range(self.n_groups)]
             resid_host = [host(resid[g], self._gidx(g)) for g in range(self.n_groups)]
-        if ring is None:
+        if explicit is not None:
+            cb.cb_extrapolate_weights(self.plan, explicit, out_t, CB[out_dtype], resid, CB[resid_dtype])
+        elif ring is None:
             cb.cb_extrapolate(self.plan, t, out_t, CB[out_dtype], resid, CB[resid_dtype])
         else:
             slot_t, head = ring
@@ -149,12 +151,14 @@ class Walk:
         return self.idx[i]
 
     def expected_and_compare(self, t, out_t, resid, resid_host, out_dtype="bf16", resid_dtype="bf16",
-                             times=None, nthreads=8):
-        """Oracle expectation for the live FIFO (or ``times`` relabelling it) and the comparison."""
+                             times=None, nthreads=8, wts=None):
+        """Oracle expectation for the live FIFO (or ``times`` relabelling it, or the
+        explicit weights ``wts``) and the comparison."""
         w = self.w
         entries = self.H.entries()
         times = times if times is not None else [e[0] for e in entries]
-        wts = orc.weights(times, t, w.t_min, w.t_max)
+        if wts is None:
+            wts = orc.weights(times, t, w.t_min, w.t_max)
         cdt = ORC[self.cdt]
         stats_out, stats_res = [], []
         items = []

@@ -134,6 +134,10 @@ def test_validation_before_launch(cb):
     assert st("cb_plan_set_option", p, cb.CB_OPT_KERNEL, 7) == cb.CB_ERR_ARG
     assert st("cb_plan_set_option", p, cb.CB_OPT_WAIT_NS, -1) == cb.CB_ERR_ARG
     assert st("cb_plan_set_option", p, 99, 0) == cb.CB_ERR_ARG
+    assert st("cb_plan_set_option", p, cb.CB_OPT_PARTIAL_HISTORY, 2) == cb.CB_ERR_ARG
+    w3 = (ctypes.c_double * 3)(0.2, 0.3, 0.5)
+    assert st("cb_extrapolate_weights", p, w3, arr(0x1000, 0x2000), 0, None, 0, None) == cb.CB_ERR_HISTORY_NOT_FULL
+    assert st("cb_extrapolate_weights", p, None, arr(0x1000, 0x2000), 0, None, 0, None) == cb.CB_ERR_ARG
     for k in (cb.CB_KERNEL_DIRECT, cb.CB_KERNEL_BULK, cb.CB_KERNEL_AUTO):
         cb.cb_plan_set_option(p, cb.CB_OPT_KERNEL, k)
     # nothing has run since binding: the status read touches no device memory
@@ -185,3 +189,18 @@ def test_export_weights_edge_cases(cb, orc):
         cb.cb_plan_export_weights(p, [650.0], 4)  # only 3 nodes precede it
     assert e.value.status == cb.CB_ERR_HISTORY_NOT_FULL
     cb.cb_plan_destroy(p)
+
+
+def test_taylor_weights_match_oracle(cb, orc):
+    rng = np.random.default_rng(23)
+    for _ in range(200):
+        n = int(rng.integers(1, 9))
+        h = float(rng.uniform(0.1, 50) * rng.choice([-1, 1]))
+        x = float(rng.uniform(-500, 500)) + h * np.arange(n)
+        xq = x[-1] + h * float(rng.uniform(0.05, 3))
+        ref = orc.taylor_weights(x, xq)
+        assert np.max(np.abs(cb.cb_taylor_weights(x, xq) - ref)) <= 1e-12 * np.abs(ref).sum()
+    with pytest.raises(cb.CbError):
+        cb.cb_taylor_weights([0.0, 1.0, 3.0], 4.0)  # not equispaced
+    with pytest.raises(cb.CbError):
+        cb.cb_taylor_weights([], 1.0)

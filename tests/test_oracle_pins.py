@@ -242,6 +242,24 @@ def test_affine_invariance(orc):
         assert _rel(orc.lagrange_basis(a * x + b, a * xq + b), orc.lagrange_basis(x, xq)) <= 1e-9
 
 
+def test_taylor_weights_golden_and_properties(orc):
+    for lhs, rhs in _rows("taylor_weights.txt"):
+        n, theta = int(lhs[0]), float(lhs[1])
+        x = np.arange(n, dtype=float)
+        g = np.array([float(v) for v in rhs])
+        assert _rel(orc.taylor_weights(x, n - 1 + theta), g) <= 1e-14, lhs
+    rng = np.random.default_rng(22)
+    for _ in range(100):
+        n = int(rng.integers(1, 9))
+        h = float(rng.uniform(0.1, 3) * rng.choice([-1, 1]))
+        x = float(rng.uniform(-5, 5)) + h * np.arange(n)
+        xq = x[-1] + h * float(rng.uniform(0, 3))
+        w = orc.taylor_weights(x, xq)
+        assert abs(w.sum() - 1) <= 1e-12 * np.abs(w).sum()  # constants are reproduced
+        if n >= 2:  # and straight lines: every backward difference beyond the first vanishes
+            assert abs(w @ x - xq) <= 1e-10 * (np.abs(w) @ np.abs(x) + abs(xq))
+
+
 def test_target_on_node_and_duplicates(orc):
     x = np.array([-1.0, -0.2, 0.5, 0.9])
     for j in range(4):
@@ -381,3 +399,34 @@ def test_pins_catch_planted_mistakes(orc):
 
     for bad in (sign_flip, reversed_order, dropped_node, wrong_target, no_normalisation):
         assert _weight_pins(bad, orc), bad.__name__
+
+
+def test_runge_study_report(orc):
+    """Sec. 3.2 / Fig. 4: extrapolating f(x) = 1 / (1 + 25 x^2) from K nodes on
+    [-1, 1] beyond x = 1 with equispaced nodes, Chebyshev roots, Chebyshev
+    extrema, and truncated Taylor (equispaced). Reported, not a gate: the
+    paper's ordering (equispaced ahead of Chebyshev roots far out) is only
+    qualitative. Checked here: the table is finite, equispaced and extrema
+    nodes coincide for K = 3, and every family interpolates the nodes."""
+    f = lambda x: 1.0 / (1.0 + 25.0 * x * x)
+    lines = []
+    for K in (3, 4, 5, 6, 8):
+        j = np.arange(1, K + 1)
+        fam = {"equispaced": np.linspace(-1, 1, K),
+               "cheb-roots": np.sort(np.cos((2 * j - 1) * np.pi / (2 * K))),
+               "cheb-extrema": np.sort(np.cos((j - 1) * np.pi / (K - 1)))}
+        row = []
+        for xq in (1.05, 1.25, 1.5, 2.0):
+            errs = {k: abs(f(xq) - orc.lagrange_basis(x, xq) @ f(x)) for k, x in fam.items()}
+            eq = fam["equispaced"]
+            errs["taylor"] = abs(f(xq) - orc.taylor_weights(eq, xq) @ f(eq))
+            assert all(np.isfinite(v) for v in errs.values())
+            row.append(" ".join(f"{k}={v:.3g}" for k, v in errs.items()))
+        lines.append(f"K={K}: " + " | ".join(row))
+        for x in fam.values():
+            for i, xi in enumerate(x):
+                e = np.zeros(K)
+                e[i] = 1.0
+                assert np.allclose(orc.lagrange_basis(x, xi), e)
+    assert np.allclose(np.linspace(-1, 1, 3), np.sort(np.cos(np.arange(3) * np.pi / 2)))
+    print("\n".join(lines))
