@@ -33,7 +33,8 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "extrapolation GB/s & % of HBM peak; µs per skipped step (all blocks), 1 GB300"
-KERNEL_SOURCES = ["paper_2608_23429_gb300/csrc/extrapolate_bulk.cu", "paper_2608_23429_gb300/csrc/extrapolate.cu",
+KERNEL_SOURCES = ["paper_2608_23429_gb300/csrc/extrapolate_bulk.cu", "paper_2608_23429_gb300/csrc/bulk_kernel.cuh",
+                  "paper_2608_23429_gb300/csrc/extrapolate.cu", "paper_2608_23429_gb300/csrc/direct_kernel.cuh",
                   "paper_2608_23429_gb300/csrc/cb_math.cuh", "paper_2608_23429_gb300/csrc/cb_device.h"]
 
 
@@ -279,15 +280,65 @@ def run_ours(args):
     slot_elems = sum(t.numel for t in w.tensors)
     esz = 2 if w.cache_dtype == "bf16" else 4
     fused = w.fused if args.fused == "auto" else args.fused == "on"
+    fused = fused or args.gated  # gates act on the hidden-state update only
     n_groups = cb.cb_plan_num_groups(plan)
     resid = [wl.hidden_state(w, g, dev) for g in range(n_groups)] if fused else None
     resid_elems = sum(w.group_numel(g) for g in range(n_groups)) if fused else 0
     # K slot reads + one output write (+ hidden state read and write)
     bytes_step = slot_elems * esz * (K + 1) + resid_elems * 2 * 2
     t_targets = [w.timesteps[s] for s in targets]
+    gates = None
+    if args.gated or args.step == "full-fused":
+        cb.cb_plan_set_shapes(plan, [t.shape for t in w.tensors])
+    if args.gated:  # per-(batch, channel) gates of each branch, bf16
+        gg = torch.Generator(device=dev).manual_seed(7)
+        gates = [(0.5 * torch.randn(t.shape[0], t.shape[-1], generator=gg, device=dev)).to(torch.bfloat16)
+                 for t in w.tensors]
+        bytes_step += sum(t.shape[0] * t.shape[-1] * 2 for t in w.tensors) if fused else 0
+    kernel_name = "extrapolate_kernel" if args.kernel == "direct" else "extrapolate_bulk_kernel"
+    # persistent buffers: their pointer arrays are built once, as a serving loop would
+    outs_p = cb.ptr_array(outs)
+    resid_p = cb.ptr_array(resid) if resid is not None else None
+    gates_p = cb.ptr_array(gates) if gates is not None else None
 
-    def step(k):
-        cb.cb_extrapolate(plan, t_targets[k % len(t_targets)], outs, cdt, resid, cb.CB_BF16, stream=stream)
+    if args.step == "skip":
+        def step(k):
+            t = t_targets[k % len(t_targets)]
+            if gates is not None:
+                cb.cb_extrapolate_gated(plan, t, outs_p, cdt, resid_p, cb.CB_BF16, gates_p, cb.CB_BF16,
+                                        stream=stream)
+            else:
+                cb.cb_extrapolate(plan, t, outs_p, cdt, resid_p, cb.CB_BF16, stream=stream)
+    else:
+        # a full step's cache write (row a4), optionally with the fused epilogue:
+        # the features come from one generated full step, re-pushed with fresh times
+        fdt = torch.float32 if args.feat_dtype == "fp32" else tdt
+        src = [wl.trajectory(w, i, w.timesteps[pushed[-1]], pushed[-1], dev, out_dtype=fdt)
+               for i in range(len(w.tensors))]
+        sdt = cb.CB_FP32 if fdt == torch.float32 else cb.CB_BF16
+        bytes_step = slot_elems * (fdt.itemsize + esz)
+        if args.step == "full-fused":
+            if resid is None:
+                resid = [wl.hidden_state(w, g, dev) for g in range(n_groups)]
+                resid_elems = sum(w.group_numel(g) for g in range(n_groups))
+            bytes_step += resid_elems * 2 * 2 + (sum(t.shape[0] * t.shape[-1] * 2 for t in w.tensors)
+                                                 if gates is not None else 0)
+        cb.cb_plan_reset(plan)
+        t0 = w.timesteps[0]
+        span = (w.timesteps[-1] - w.timesteps[0]) / (args.warmup + args.steps + 1)
+        times = iter([t0 + span * i for i in range(args.warmup + args.steps + 1)])
+        # the fused epilogue runs the skipped-step kernel on a one-entry history
+        kernel_name = "push_kernel" if args.step == "full" else kernel_name
+        src_p = cb.ptr_array(src)
+        resid_p = cb.ptr_array(resid) if resid is not None else None
+
+        def step(k):
+            t = next(times)
+            if args.step == "full":
+                cb.cb_cache_push(plan, src_p, sdt, t, stream=stream)
+            else:
+                cb.cb_cache_push_residual(plan, src_p, sdt, t, resid_p, cb.CB_BF16, gates_p, cb.CB_BF16,
+                                          stream=stream)
 
     for k in range(args.warmup):
         step(k)
@@ -300,11 +351,13 @@ def run_ours(args):
         t_all0 = torch.cuda.Event(enable_timing=True)
         t_all1 = torch.cuda.Event(enable_timing=True)
         t_all0.record(stream)
+        h0 = time.perf_counter()
         for k in range(args.steps):
             ev[k][0].record(stream)
             step(k)
             ev[k][1].record(stream)
         t_all1.record(stream)
+        host_ms = (time.perf_counter() - h0) * 1e3 / args.steps  # submission time per step
         stream.synchronize()
         torch.cuda.synchronize()
         if ws > 1:
@@ -326,11 +379,11 @@ def run_ours(args):
     # cached feature sets from pinned host memory (push), extrapolate, read the
     # predictions back; every copy is inside the timed region.
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and args.step == "skip" and not args.gated:
         e2e = run_e2e(args, torch, cb, wl, w, plan, cdt, tdt, dev, pushed, t_targets, bytes_step, ws, fused)
 
     cpu = None
-    if rank == 0 and ws == 1 and not args.no_cpu:
+    if rank == 0 and ws == 1 and not args.no_cpu and args.step == "skip":
         host, wts, ti = sample_host_features(w, torch, wl, orc, args.cpu_elems, dev)
         threads = os.cpu_count() or 1
         gbs, n, reps, el = cpu_oracle_run(w, host, wts, args.cpu_seconds, threads)
@@ -341,20 +394,23 @@ def run_ours(args):
     cb.cb_plan_destroy(plan)
     if rank == 0:
         desc = workload_description(w)
-        desc.update({"bytes_per_step": bytes_step, "fused_residual": fused, "targets": targets,
+        desc.update({"bytes_per_step": bytes_step, "fused_residual": fused, "step": args.step,
+                     "gated": bool(args.gated), "targets": targets,
                      "history_steps": pushed[-K:],
                      "l2": "inputs larger than L2 (no flush)", "launch": "1 grouped persistent kernel per step",
                      "parallelism": f"replicas x{ws}" if ws > 1 else "1 GPU"})
         line = {
             "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(ms_step, 4),
-            "us_per_step": round(ms_step * 1e3, 2), "pct_hbm_peak": round(100 * value / ws / peak, 2),
+            "us_per_step": round(ms_step * 1e3, 2), "host_us_per_step": round(host_ms * 1e3, 2),
+            "pct_hbm_peak": round(100 * value / ws / peak, 2),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
             "data": "synthetic", "config": desc,
             "roofline": {"bound": "hbm", "achieved": round(achieved, 2), "peak": peak, "unit": "GB/s",
                          "frac": round(achieved / peak, 4), "peak_source": peak_src,
-                         "traffic": recorded_traffic(args.config) if args.scale == 1 else None,
-                         "kernel": "extrapolate_kernel" if args.kernel == "direct" else "extrapolate_bulk_kernel",
+                         "traffic": (recorded_traffic(args.config) if args.scale == 1 and args.step == "skip"
+                                     and not args.gated else None),
+                         "kernel": kernel_name,
                          "avg_launch_us": round(avg_kern * 1e3, 2)},
             "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks, "gpu_launches": args.steps,
         }
@@ -453,6 +509,12 @@ def main():
                     help="add the predictions into the blocks' hidden states (auto: as the workload states)")
     ap.add_argument("--e2e-mode", default="zerocopy", choices=["zerocopy", "copy"],
                     help="e2e host buffers: read/written by the kernels over C2C, or staged by copies")
+    ap.add_argument("--step", default="skip", choices=["skip", "full", "full-fused"],
+                    help="skip: a skipped step (the metric); full: a full step's cache write; "
+                         "full-fused: the cache write with the hidden-state update")
+    ap.add_argument("--gated", action="store_true", help="per-(batch, channel) gates on the hidden-state update")
+    ap.add_argument("--feat-dtype", default="bf16", choices=["bf16", "fp32"],
+                    help="type of the full step's features (--step full / full-fused)")
     ap.add_argument("--kernel", default="auto", choices=["auto", "direct", "bulk"],
                     help="skipped-step kernel variant (both compute identical bits)")
     ap.add_argument("--scale", type=int, default=1,

@@ -182,6 +182,41 @@ int cb_extrapolate_ring(cb_plan* plan, const double* slot_t, int head, double t_
                         void* const* outs, cb_dtype out_dtype, void* const* resid,
                         cb_dtype resid_dtype, void* stream);
 
+/* Shapes of the branch tensors, needed by the gated calls: bth[3*i + 0..2] =
+ * batch, tokens, hidden of tensor i (their product must be its numel;
+ * tokens * hidden < 2^32). Tensors of one residual group must share tokens
+ * and hidden. Errors: CB_ERR_ARG, CB_ERR_LIMIT. */
+int cb_plan_set_shapes(cb_plan* plan, const int64_t* bth);
+
+/* Skipped step with gated hidden-state updates. DiT blocks add each branch
+ * through a per-sample, per-channel gate computed from the timestep
+ * conditioning (the adaptive normalisation of the blocks, Sec. 3.1); when the
+ * cache holds the un-gated branch outputs, the gate of the current step
+ * multiplies the prediction:
+ *     resid[g] <- round(resid[g] + sum_{i in g} gate_i[b, h] * P_i[b, tok, h]).
+ * gates: host array of n_tensors pointers (NULL array or entries: gate 1),
+ * each a [batch, hidden] array of gate_dtype broadcast over tokens; shapes
+ * must be set (cb_plan_set_shapes). Predictions written to outs stay
+ * un-gated. Otherwise as cb_extrapolate; errors as cb_extrapolate. */
+int cb_extrapolate_gated(cb_plan* plan, double t_target, void* const* outs, cb_dtype out_dtype,
+                         void* const* resid, cb_dtype resid_dtype, const void* const* gates,
+                         cb_dtype gate_dtype, void* stream);
+
+/* Full step with its epilogue fused (Sec. 3.3 / Alg. 1, full-computation
+ * branch, plus the block residual of Sec. 3.1): one pass stores every branch
+ * output in H exactly as cb_cache_push does and, for each residual group g
+ * with resid[g] non-NULL, adds the un-rounded outputs into the hidden state:
+ *     resid[g] <- round(resid[g] + sum_{i in g} gate_i * feats_i)
+ * (one rounding of the un-rounded sum, with the accuracy of cb_extrapolate's
+ * hidden-state update; gates as in cb_extrapolate_gated, may be NULL). It runs
+ * the skipped-step kernels on a one-entry history of weight 1 (the features
+ * themselves), so it saves the separate read of the features that the
+ * residual add would otherwise need. Errors: as cb_cache_push, plus those of
+ * the gates. */
+int cb_cache_push_residual(cb_plan* plan, const void* const* feats, cb_dtype feat_dtype, double t,
+                           void* const* resid, cb_dtype resid_dtype, const void* const* gates,
+                           cb_dtype gate_dtype, void* stream);
+
 /* Skipped step with caller-chosen weights: P_i = sum_j w_logical[j] F_{i,j}
  * over the live history (the kernel of cb_extrapolate with the weights of
  * Sec. 3.3's linear combination given directly, e.g. another node family's

@@ -56,6 +56,8 @@ def lib():
         L.orc_convert.argtypes, L.orc_convert.restype = [P, I, I64, P, I], None
         L.orc_extrapolate.argtypes = [I, I, P, I, P, P, I, I64, P, I, P, I, I]
         L.orc_extrapolate.restype = I
+        L.orc_extrapolate_gated.argtypes = [I, I, P, I, P, P, I, I64, P, I, P, I, P, I]
+        L.orc_extrapolate_gated.restype = I
         _lib = L
     return _lib
 
@@ -153,9 +155,10 @@ def weights(node_t, t_target: float, t_min: float, t_max: float) -> np.ndarray:
 
 # ------------------------------------------------------------- extrapolation
 def extrapolate(F, w, f_dtype: int, out_dtype: int | None = None, X=None, x_dtype: int = FP32,
-                resid_dtype: int | None = None, nthreads: int = 1):
+                resid_dtype: int | None = None, nthreads: int = 1, G=None):
     """Per element: P_b = sum_j w_j F[b][j] (fp64) rounded once to ``out_dtype``;
-    with ``resid_dtype`` set, also X + sum_b P_b rounded once.
+    with ``resid_dtype`` set, also X + sum_b G_b P_b rounded once (G_b: optional
+    per-element gates, 1 where absent).
 
     ``F`` is a list over branches b of lists over history entries j (oldest first),
     each a flat array of the same length in ``f_dtype`` (bf16 as uint16 bits).
@@ -175,11 +178,17 @@ def extrapolate(F, w, f_dtype: int, out_dtype: int | None = None, X=None, x_dtyp
         optrs = (ctypes.c_void_p * nb)(*[o.ctypes.data for o in outs])
     xa = None if X is None else np.ascontiguousarray(X, dtype=_NP[x_dtype]).ravel()
     resid = None if resid_dtype is None else np.empty(n, dtype=_NP[resid_dtype])
-    rc = lib().orc_extrapolate(
+    garr = None
+    gptrs = None
+    if G is not None:  # per-member gates expanded to the element space (fp64), None = 1
+        garr = [None if g is None else _f64(g).ravel() for g in G]
+        assert all(g is None or g.size == n for g in garr)
+        gptrs = (ctypes.c_void_p * nb)(*[None if g is None else g.ctypes.data for g in garr])
+    rc = lib().orc_extrapolate_gated(
         K, nb, fptrs, f_dtype, _ptr(w), None if xa is None else _ptr(xa), x_dtype, n,
         optrs, out_dtype if out_dtype is not None else FP64,
         None if resid is None else _ptr(resid), resid_dtype if resid_dtype is not None else FP64,
-        int(nthreads))
+        gptrs, int(nthreads))
     if rc != 0:
         raise RuntimeError(f"orc_extrapolate failed ({rc})")
     return outs, resid

@@ -27,7 +27,8 @@
  *                       f_t = sum_j w_j f_{s_j}, per element, in fp64, then one
  *                       rounding to the output type; optionally the block
  *                       residual of Sec. 3.1 (B(x) = x + S + C + M): the hidden
- *                       state plus every branch prediction, rounded once.
+ *                       state plus every branch prediction, each optionally
+ *                       times its per-element gate, rounded once.
  *   orc_convert         the cache write of Alg. 1 ("store the pair in H"):
  *                       a copy, or fp32 -> bf16 round-to-nearest-even.
  *   orc_bf16_encode /   bf16 <-> fp64 from the IEEE-754 bit layout (8 exponent
@@ -217,6 +218,7 @@ typedef struct {
     int out_dtype;
     void* resid_out; /* NULL when no residual is written */
     int resid_dtype;
+    const double* const* G; /* nb per-element gate arrays (NULL array or entry: 1) */
     int64_t begin, end;
 } orc_job;
 
@@ -228,16 +230,27 @@ static void* orc_extrapolate_range(void* arg) {
             double p = 0.0;
             for (int j = 0; j < J->K; ++j) p += J->w[j] * load_elem(J->F[b * J->K + j], J->f_dtype, e);
             if (J->outs && J->outs[b]) store_elem(J->outs[b], J->out_dtype, e, p);
-            total += p;
+            total += (J->G && J->G[b]) ? J->G[b][e] * p : p; /* gated residual, Sec. 3.1 */
         }
         if (J->resid_out) store_elem(J->resid_out, J->resid_dtype, e, total);
     }
     return NULL;
 }
 
+int orc_extrapolate_gated(int K, int nb, const void* const* F, int f_dtype, const double* w,
+                          const void* X, int x_dtype, int64_t n, void* const* outs, int out_dtype,
+                          void* resid_out, int resid_dtype, const double* const* G, int nthreads);
+
 int orc_extrapolate(int K, int nb, const void* const* F, int f_dtype, const double* w,
                     const void* X, int x_dtype, int64_t n, void* const* outs, int out_dtype,
                     void* resid_out, int resid_dtype, int nthreads) {
+    return orc_extrapolate_gated(K, nb, F, f_dtype, w, X, x_dtype, n, outs, out_dtype, resid_out,
+                                 resid_dtype, NULL, nthreads);
+}
+
+int orc_extrapolate_gated(int K, int nb, const void* const* F, int f_dtype, const double* w,
+                          const void* X, int x_dtype, int64_t n, void* const* outs, int out_dtype,
+                          void* resid_out, int resid_dtype, const double* const* G, int nthreads) {
     if (K <= 0 || nb <= 0 || !F || !w || n < 0) return -1;
     if (nthreads < 1) nthreads = 1;
     if (nthreads > 256) nthreads = 256;
@@ -248,7 +261,7 @@ int orc_extrapolate(int K, int nb, const void* const* F, int f_dtype, const doub
         orc_job* J = &jobs[t];
         J->K = K; J->nb = nb; J->F = F; J->f_dtype = f_dtype; J->w = w;
         J->X = X; J->x_dtype = x_dtype; J->outs = outs; J->out_dtype = out_dtype;
-        J->resid_out = resid_out; J->resid_dtype = resid_dtype;
+        J->resid_out = resid_out; J->resid_dtype = resid_dtype; J->G = G;
         J->begin = t * chunk < n ? t * chunk : n;
         J->end = (t + 1) * chunk < n ? (t + 1) * chunk : n;
     }

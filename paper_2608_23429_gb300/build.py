@@ -20,7 +20,8 @@ LIB = os.path.join(HERE, "libchebboost.so")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["extrapolate.cu", "extrapolate_bulk.cu", "push.cu", "plan.cpp"]
+SOURCES = ["extrapolate.cu", "extrapolate_gated.cu", "extrapolate_bulk.cu", "extrapolate_bulk_gated.cu",
+           "push.cu", "plan.cpp"]
 
 
 def _nvcc() -> str:

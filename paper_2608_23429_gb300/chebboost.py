@@ -48,6 +48,9 @@ _sig = {
     "cb_extrapolate": ([_P, _D, _PP, _I, _PP, _I, _P], _I),
     "cb_extrapolate_ring": ([_P, _P, _I, _D, _PP, _I, _PP, _I, _P], _I),
     "cb_extrapolate_weights": ([_P, _P, _PP, _I, _PP, _I, _P], _I),
+    "cb_plan_set_shapes": ([_P, _P], _I),
+    "cb_extrapolate_gated": ([_P, _D, _PP, _I, _PP, _I, _PP, _I, _P], _I),
+    "cb_cache_push_residual": ([_P, _PP, _I, _D, _PP, _I, _PP, _I, _P], _I),
     "cb_weights": ([_P, _D, _P], _I),
     "cb_taylor_weights": ([_P, _I, _D, _P], _I),
     "cb_plan_export_weights": ([_P, _P, _I, _P], _I),
@@ -90,10 +93,17 @@ def _addr(x) -> int | None:
     return int(x.data_ptr())
 
 
-def _ptr_array(xs):
-    if xs is None:
-        return None
+def ptr_array(xs):
+    """The pointer array of a list of buffers (tensors, ints or None), in the
+    form every call below also accepts: a loop over persistent buffers builds
+    it once instead of on every call."""
     return (ctypes.c_void_p * len(xs))(*[_addr(x) for x in xs])
+
+
+def _ptr_array(xs):
+    if xs is None or isinstance(xs, ctypes.Array):
+        return xs
+    return ptr_array(xs)
 
 
 def _stream(s):
@@ -158,6 +168,26 @@ def cb_extrapolate_weights(plan, w_logical, outs, out_dtype: int, resid=None, re
     w = _f64(w_logical)
     _check(_lib.cb_extrapolate_weights(plan, w.ctypes.data, _ptr_array(outs), out_dtype, _ptr_array(resid),
                                        resid_dtype, _stream(stream)), "cb_extrapolate_weights")
+
+
+def cb_plan_set_shapes(plan, shapes) -> None:
+    """``shapes``: sequence of (batch, tokens, hidden), one per tensor."""
+    bth = np.ascontiguousarray(np.asarray(shapes, dtype=np.int64).reshape(-1))
+    _check(_lib.cb_plan_set_shapes(plan, bth.ctypes.data), "cb_plan_set_shapes")
+
+
+def cb_extrapolate_gated(plan, t_target: float, outs, out_dtype: int, resid, resid_dtype: int, gates,
+                         gate_dtype: int = CB_BF16, stream=None) -> None:
+    _check(_lib.cb_extrapolate_gated(plan, float(t_target), _ptr_array(outs), out_dtype, _ptr_array(resid),
+                                     resid_dtype, _ptr_array(gates), gate_dtype, _stream(stream)),
+           "cb_extrapolate_gated")
+
+
+def cb_cache_push_residual(plan, feats, feat_dtype: int, t: float, resid, resid_dtype: int = CB_BF16,
+                           gates=None, gate_dtype: int = CB_BF16, stream=None) -> None:
+    _check(_lib.cb_cache_push_residual(plan, _ptr_array(feats), feat_dtype, float(t), _ptr_array(resid),
+                                       resid_dtype, _ptr_array(gates), gate_dtype, _stream(stream)),
+           "cb_cache_push_residual")
 
 
 def cb_weights(plan, t_target: float, n: int) -> np.ndarray:

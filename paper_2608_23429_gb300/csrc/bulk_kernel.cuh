@@ -1,0 +1,369 @@
+// Skipped-step kernel, bulk-copy pipeline variant (same arithmetic and bits as
+// extrapolate.cu; Sec. 3.3, Eq. for f_t; Alg. 1, extrapolation branch).
+//
+// One CTA per SM. A producer lane moves, for every work unit (one tile of one
+// branch tensor), the K history chunks of 8 KB each from HBM into a ring of
+// shared-memory stages with cp.async.bulk (the Blackwell bulk-copy engine),
+// each stage guarded by a "full" mbarrier (transaction bytes) and an "empty"
+// mbarrier (one arrival per consumer warp). Consumer warps read their 8-element
+// vectors of the K chunks from shared memory, release the stage, and compute
+// and store from registers. With S stages of K x 8 KB (S = 5 for K = 5) up to
+// ~160 KB per SM stay in flight independently of the consumers' registers,
+// which is what bounds the direct-load variant.
+//
+// Every consumer thread takes one 8-element vector of a tile: 16 consumer
+// warps for bf16 tiles (17 warps, up to 96 registers per thread), 8 for fp32
+// tiles. Many warps per scheduler hide the consumers' fixed latencies; the
+// arithmetic per byte is high enough that 8 warps with two vectors each
+// leave the grouped launches issue-bound. Two kinds of launch (GROUPED):
+//   * predictions only: each stage is released as soon as it is in
+//     registers, and guarded elements are recomputed from registers;
+//   * with hidden states: stages are released after the member's arithmetic,
+//     guarded elements are recomputed from shared memory (so the history
+//     values die early). The producer also stages each tile's bf16 hidden
+//     state (one more chunk with the group's last member) and the consumers
+//     hold the group's member stages until the hidden state is written (the
+//     host guarantees more stages than members, so holding cannot starve the
+//     producer). With gates, each member's stage also carries the gate rows
+//     of the batches its tile touches, so that no consumer waits on a global
+//     load.
+//
+// Every wait is bounded (%globaltimer). A wait that runs out records a code in
+// the plan's device status word and the thread returns; the producer then
+// waits, with its own limit (at least 10 ms), for the copies it has issued
+// before it exits. A test option makes the producer announce the first unit's
+// bytes without issuing its copies, so that the consumers' wait runs out with
+// no fault and nothing in flight.
+#pragma once
+
+#include "cb_math.cuh"
+
+namespace cbk {
+namespace {
+
+// One 8-element vector per consumer thread and tile: 16 consumer warps for
+// bf16 tiles (512 vectors), 8 for fp32 tiles (256 vectors).
+template <bool CB16>
+struct Shape {
+    static constexpr int consumer_warps = CB16 ? 16 : 8;
+    static constexpr int consumers = consumer_warps * 32;
+    static constexpr int threads = consumers + 32;  // plus the producer warp
+};
+constexpr int kChunkBytes = 8192;   // one history entry's share of a tile
+constexpr int kBarrierBytes = 256;  // full[S] and empty[S] barriers, S <= 16
+constexpr unsigned long long kMinDrainNs = 10000000ull;  // copies land in microseconds
+constexpr unsigned long long kMaxWaitNs = 60000000000ull;  // no wait outlives a minute
+
+__device__ __forceinline__ uint32_t smem_addr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ unsigned long long now_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Wait for the phase with the given parity to complete, for at most limit_ns
+// (never more than kMaxWaitNs).
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, unsigned long long limit_ns) {
+    if (limit_ns > kMaxWaitNs) limit_ns = kMaxWaitNs;
+    if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = now_ns();
+    while (!mbar_try_wait(bar, parity))
+        if (now_ns() - t0 > limit_ns) return false;
+    return true;
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+
+// Global -> shared bulk copy completing `bytes` transaction bytes on `bar`.
+// dst, src 16-byte aligned; bytes a multiple of 16.
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     dst),
+                 "l"(src), "r"(bytes), "r"(bar)
+                 : "memory");
+}
+
+__device__ __forceinline__ void record(int* status, int code) {
+    if (status) atomicOr(status, code);
+}
+
+// GROUPED: some item updates a hidden state (stage holding, hidden-state
+// staging, 8 consumer warps); prediction-only launches compile without that
+// bookkeeping and with 16 consumer warps. GATED (with GROUPED): the hidden
+// state receives g_b * P_b, with a per-(batch, channel) gate per member.
+template <int K, bool CB16, bool GROUPED, bool GATED>
+__global__ void __launch_bounds__(Shape<CB16>::threads, 1)
+    extrapolate_bulk_kernel(const __grid_constant__ ExtrapArgs A) {
+    extern __shared__ __align__(128) unsigned char smem[];
+    constexpr int NCW = Shape<CB16>::consumer_warps;
+    constexpr int NCT = Shape<CB16>::consumers;
+    constexpr long long TE = tile_elems(CB16);  // 8 KB per history chunk for both cache types
+    constexpr int ES = CB16 ? 2 : 4;
+    constexpr int NV = (int)(TE / kVecElems);     // vectors per tile: 512 (bf16) or 256 (fp32)
+    constexpr int U = NV >= NCT ? NV / NCT : 1;   // vectors per consumer thread per tile
+    static_assert(NV % NCT == 0 || NCT % NV == 0, "vectors spread evenly over the consumers");
+    static_assert(TE * ES == kChunkBytes, "one tile of one history entry is one chunk");
+    const int S = A.stages;
+    const uint32_t full0 = smem_addr(smem);
+    const uint32_t empty0 = full0 + 8u * (uint32_t)S;
+    const uint32_t buf0 = smem_addr(smem + kBarrierBytes);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(full0 + 8u * s, 1);
+            mbar_init(empty0 + 8u * s, NCW);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncthreads();
+
+    const int C = GROUPED ? A.stage_chunks : K;
+    const uint32_t stage_bytes = (uint32_t)C * kChunkBytes + (GATED ? A.stage_gate_bytes : 0u);
+    if (warp == NCW) {  // ---------------------------------- producer
+        if (lane != 0) return;
+        int it = 0;
+        unsigned u = 0;
+        bool ok = true;
+        for (int tile = blockIdx.x; ok && tile < A.tiles_total; tile += gridDim.x) {
+            while (tile >= A.tile_begin[it + 1]) ++it;
+            const long long numel = A.numel[it];
+            const long long e0 = (long long)(tile - A.tile_begin[it]) * TE;
+            // consumers read shared memory only for whole tiles of aligned items;
+            // for the ragged last tile (or a misaligned item) the stage is
+            // cycled without data and they recompute from global memory
+            const bool full_tile = A.vec_ok[it] && e0 + TE <= numel;
+            const uint32_t bytes = full_tile ? (uint32_t)kChunkBytes : 0u;
+            const int first = A.first[it];
+            const int nb = GROUPED ? A.nb[it] : 1;
+            const unsigned char* resid = GROUPED ? reinterpret_cast<const unsigned char*>(A.resid[it]) : nullptr;
+            // gate rows b0..b1 of the batches this tile touches (b1 <= b0 + 1:
+            // the host stages gates only when a batch holds a tile or more)
+            uint32_t gbytes = 0;
+            size_t gsrc = 0;
+            if (GATED && A.stage_gate_bytes && resid && full_tile && A.i_row[it] != 0) {
+                const long long row = A.i_row[it];
+                const long long b0 = e0 / row, b1 = (e0 + TE - 1) / row;
+                const size_t gs = A.gate_bf16 ? 2 : 4;
+                gsrc = (size_t)b0 * A.i_hidden[it] * gs;
+                gbytes = (uint32_t)((b1 - b0 + 1) * A.i_hidden[it] * gs);
+            }
+            for (int m = 0; m < nb; ++m, ++u) {
+                const uint32_t stage = u % (unsigned)S, q = u / (unsigned)S;
+                if (q > 0 && !mbar_wait(empty0 + 8u * stage, (q - 1) & 1u, A.wait_ns)) {
+                    record(A.status, 2);
+                    ok = false;
+                    break;
+                }
+                // the tile's bf16 hidden state travels with its last member
+                const bool with_x = GROUPED && A.stage_x && resid && full_tile && m == nb - 1;
+                const uint32_t xbytes = with_x ? (uint32_t)(TE * 2) : 0u;
+                const uint32_t gb = (GATED && A.m_gate[first + m]) ? gbytes : 0u;
+                mbar_expect_tx(full0 + 8u * stage, (uint32_t)K * bytes + xbytes + gb);
+                if (A.withhold_first && u == 0) continue;
+                const uint32_t dst = buf0 + stage * stage_bytes;
+                if (bytes) {
+#pragma unroll
+                    for (int j = 0; j < K; ++j)
+                        bulk_g2s(dst + j * (uint32_t)kChunkBytes, hist_ptr(A, j, A.m_off[first + m]) + e0 * ES, bytes,
+                                 full0 + 8u * stage);
+                }
+                if (xbytes) bulk_g2s(dst + K * (uint32_t)kChunkBytes, resid + e0 * 2, xbytes, full0 + 8u * stage);
+                if (gbytes && A.m_gate[first + m])
+                    bulk_g2s(dst + C * (uint32_t)kChunkBytes,
+                             reinterpret_cast<const unsigned char*>(A.m_gate[first + m]) + gsrc, gbytes,
+                             full0 + 8u * stage);
+            }
+        }
+        // never leave while copies into this CTA's shared memory are in flight
+        const unsigned long long drain_ns = A.wait_ns > kMinDrainNs ? A.wait_ns : kMinDrainNs;
+        for (unsigned q = u > (unsigned)S ? u - S : 0; q < u; ++q)
+            if (!mbar_wait(full0 + 8u * (q % S), (q / S) & 1u, drain_ns)) {
+                record(A.status, 4);
+                break;
+            }
+        return;
+    }
+
+    // ------------------------------------------------------------ consumers
+    const int c = threadIdx.x;
+    const unsigned char* stages = smem + kBarrierBytes;
+    auto chunk = [&](uint32_t stage, int j) { return stages + stage * stage_bytes + (size_t)j * kChunkBytes; };
+    auto gate_stage = [&](uint32_t stage) -> const void* { return stages + stage * stage_bytes + (size_t)C * kChunkBytes; };
+    int it = 0;
+    unsigned u = 0;
+    for (int tile = blockIdx.x; tile < A.tiles_total; tile += gridDim.x) {
+        while (tile >= A.tile_begin[it + 1]) ++it;
+        const long long numel = A.numel[it];
+        const long long e0 = (long long)(tile - A.tile_begin[it]) * TE;
+        const int nb = GROUPED ? A.nb[it] : 1;
+        const int first = A.first[it];
+        void* resid = GROUPED ? A.resid[it] : nullptr;
+        // whole aligned tiles come from shared memory; the ragged last tile of a
+        // tensor and misaligned items take the compensated scalar path
+        const bool full_tile = A.vec_ok[it] && e0 + TE <= numel;
+        // with a hidden state, every member's stage stays held until the hidden
+        // state is written, so that its guarded elements can be recomputed
+        const bool hold = GROUPED && full_tile && resid != nullptr;
+        const bool mine = NV >= NCT || c < NV;  // fp32 tiles have fewer vectors than consumers
+        const unsigned u0 = u;
+        long long ev[U];
+#pragma unroll
+        for (int v = 0; v < U; ++v) ev[v] = e0 + ((long long)v * NCT + c) * kVecElems;
+        // gate offsets of this thread's vectors, relative to the gate rows the
+        // producer staged (or absolute, when gates stay in global memory)
+        unsigned gi[U];
+        if constexpr (GATED) {
+            if (hold && A.i_row[it] != 0) {  // items without a shape carry no gate
+                gate_offsets<U>(A, it, e0, ev, gi);
+                if (A.stage_gate_bytes) {
+                    const unsigned b0h = (unsigned)e0 / A.i_row[it] * A.i_hidden[it];  // gated: numel < 2^32
+#pragma unroll
+                    for (int v = 0; v < U; ++v) gi[v] -= b0h;
+                }
+            }
+        }
+        Acc<U> acc;
+        acc.zero();
+        for (int m = 0; m < nb; ++m, ++u) {
+            const uint32_t stage = u % (unsigned)S, q = u / (unsigned)S;
+            if (!mbar_wait(full0 + 8u * stage, q & 1u, A.wait_ns)) {
+                record(A.status, 1);
+                return;
+            }
+            RawVecs<K, CB16, U> raw;
+            if (full_tile && mine) {
+#pragma unroll
+                for (int v = 0; v < U; ++v)
+#pragma unroll
+                    for (int j = 0; j < K; ++j) {
+                        const unsigned char* p = chunk(stage, j) + (size_t)(ev[v] - e0) * ES;
+                        raw[v][j][0] = *reinterpret_cast<const uint4*>(p);
+                        if constexpr (!CB16) raw[v][j][CB16 ? 0 : 1] = *reinterpret_cast<const uint4*>(p + 16);
+                    }
+            }
+            // gates of this member (staged rows or global memory), read as
+            // each vector is accumulated
+            const void* gp = GATED ? A.m_gate[first + m] : nullptr;
+            if (GATED && gp && A.stage_gate_bytes) gp = gate_stage(stage);
+            auto gate = [&](int v, float (&gv)[8]) {
+                if (gp)
+                    load_x8(gp, A.gate_bf16, (long long)gi[v], gv);
+                else
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) gv[e] = 1.0f;
+            };
+            // prediction-only launches release the stage at once and recompute
+            // guarded elements from registers; grouped launches keep the stage
+            // until the member is done and recompute from shared memory, which
+            // frees the history values' registers early
+            if (!GROUPED) {
+                __syncwarp();
+                if (lane == 0) mbar_arrive(empty0 + 8u * stage);
+            }
+            if (full_tile && mine) {
+                void* out = member_out<K, CB16, U>(A, first + m, ev, raw);
+                if (A.precise) {
+                    member_precise<K, CB16, U, GATED>(A, out, ev, raw, resid != nullptr, acc, gate);
+                } else if constexpr (GROUPED) {
+                    auto exact = [&](int v, int e, float& hi, float& lo) {
+                        const size_t off = (size_t)(ev[v] - e0 + e) * ES;
+                        float p = 0.0f, cc = 0.0f;
+#pragma unroll
+                        for (int j = 0; j < K; ++j) {
+                            const unsigned char* src = chunk(stage, j) + off;
+                            const float f = CB16 ? __uint_as_float((uint32_t)(*reinterpret_cast<const uint16_t*>(src)) << 16)
+                                                 : *reinterpret_cast<const float*>(src);
+                            dot2_step(A.w_hi[j], A.w_lo[j], f, p, cc);
+                        }
+                        two_sum(p, cc, hi, lo);
+                    };
+                    member_fast<K, CB16, U, false, GATED>(A, A.m_off[first + m], out, ev, raw, resid != nullptr,
+                                                          acc, gate, exact);
+                } else {
+                    member_fast<K, CB16, U, true, GATED>(A, A.m_off[first + m], out, ev, raw, resid != nullptr,
+                                                         acc, gate);
+                }
+            }
+            if (GROUPED && !hold) {
+                __syncwarp();
+                if (lane == 0) mbar_arrive(empty0 + 8u * stage);
+            }
+        }
+        if (GROUPED && hold) {
+            const uint32_t last = (u0 + nb - 1) % (unsigned)S;
+            auto xload = [&](int v, float (&x)[8]) {
+                if (A.stage_x)
+                    unpack_bf16x8(*reinterpret_cast<const uint4*>(chunk(last, K) + (size_t)(ev[v] - e0) * 2), x);
+                else
+                    load_x8(resid, A.resid_bf16, ev[v], x);
+            };
+            if (!mine) {
+            } else if (A.precise) {
+                resid_precise<U>(A, ev, acc, resid, xload);
+            } else {
+                // Dot2 of x + sum_b P_b for one element, from the held stages
+                auto exact = [&](int v, int e, float xe, float& hi, float& lo) {
+                    const size_t off = (size_t)(ev[v] - e0 + e) * ES;
+                    float tp = xe, tc = 0.0f;
+                    for (int m = 0; m < nb; ++m) {
+                        const uint32_t st = (u0 + m) % (unsigned)S;
+                        float p = 0.0f, cc = 0.0f, h, l, qq;
+#pragma unroll
+                        for (int j = 0; j < K; ++j) {
+                            const unsigned char* src = chunk(st, j) + off;
+                            const float f = CB16 ? __uint_as_float((uint32_t)(*reinterpret_cast<const uint16_t*>(src)) << 16)
+                                                 : *reinterpret_cast<const float*>(src);
+                            dot2_step(A.w_hi[j], A.w_lo[j], f, p, cc);
+                        }
+                        two_sum(p, cc, h, l);
+                        if constexpr (GATED) {
+                            (void)qq;
+                            const void* gm = A.m_gate[first + m];
+                            float gv = 1.0f;
+                            if (gm) gv = load_elem(A.stage_gate_bytes ? gate_stage(st) : gm, A.gate_bf16, gi[v] + e);
+                            add_gated_pair(gv, h, l, tp, tc);
+                        } else {
+                            two_sum(tp, h, tp, qq);
+                            tc = __fadd_rn(tc, __fadd_rn(qq, l));
+                        }
+                    }
+                    two_sum(tp, tc, hi, lo);
+                };
+                resid_fast<K, U>(A, it, ev, acc, resid, xload, exact);
+            }
+            __syncwarp();
+            if (lane == 0)
+                for (int m = 0; m < nb; ++m) mbar_arrive(empty0 + 8u * ((u0 + m) % (unsigned)S));
+        } else if (!full_tile) {
+            const long long end = e0 + TE < numel ? e0 + TE : numel;
+            for (long long e = e0 + c; e < end; e += NCT) scalar_element<CB16>(A, K, it, e);
+        }
+    }
+}
+
+}  // namespace
+}  // namespace cbk

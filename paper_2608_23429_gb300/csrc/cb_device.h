@@ -25,7 +25,10 @@ __host__ __device__ constexpr long long tile_elems(bool cache_bf16) {
 // Every item is cut into tiles of tile_elems() elements; tiles are numbered
 // consecutively across items and dealt to a persistent grid.
 struct ExtrapArgs {
-    const unsigned char* cache;  // ring arena
+    // byte address of the history: entry j of member m starts at
+    // hist_base + slot_off[j] + m_off[m] (the ring arena and offsets inside it;
+    // for a full step's epilogue, base 0 and m_off the new features' addresses)
+    unsigned long long hist_base;
     long long slot_off[8];       // byte offset of history entry j (0 = oldest)
     float w_hi[8];               // fp32(w_j)
     float w_lo[8];               // fp32(w_j - w_hi[j])
@@ -35,9 +38,11 @@ struct ExtrapArgs {
     int out_bf16;    // predictions are bf16 (else fp32)
     int resid_bf16;  // hidden states are bf16 (else fp32)
     int precise;     // 1: compensated (Dot2) arithmetic for every element
+    int copy_out;    // full-step epilogue: outputs receive the (K = 1) sources converted, not a prediction
     int stages;                  // bulk variant: shared-memory pipeline depth
     int stage_chunks;            // bulk variant: 8 KB chunks per stage (K, or K + 1 with hidden states)
     int stage_x;                 // bulk variant: bf16 hidden states are staged as chunk K
+    unsigned stage_gate_bytes;   // bulk variant: bytes per stage for gate rows (0: gates read from global)
     unsigned long long wait_ns;  // bulk variant: limit of every barrier wait
     int* status;                 // bulk variant: device status word (codes OR-ed in)
     int withhold_first;          // bulk variant, tests only: announce but never issue the first copies
@@ -49,6 +54,11 @@ struct ExtrapArgs {
     short first[kMaxItems];           // first member index
     long long m_off[kMaxMembers];     // byte offset of the member tensor inside one slot
     void* m_out[kMaxMembers];         // prediction output of the member, or null
+    // gated hidden-state update (x <- x + sum_b g_b * P_b); read by gated kernels only
+    int gate_bf16;                      // gates are bf16 (else fp32)
+    const void* m_gate[kMaxMembers];    // gate [batch, hidden] of the member, or null (gate 1)
+    unsigned i_hidden[kMaxItems];       // hidden size of the item's tensors
+    unsigned i_row[kMaxItems];          // tokens * hidden of the item's tensors
 };
 
 // One full-step launch: copy/convert every tensor into one ring slot.
@@ -65,14 +75,21 @@ struct PushArgs {
 
 constexpr long long push_tile_elems = (long long)kThreads * 2 * kVecElems;
 
+
 cudaError_t launch_extrapolate(const ExtrapArgs& a, int K, bool cache_bf16, int grid, cudaStream_t s);
+// gated variant of the direct kernel (extrapolate_gated.cu)
+cudaError_t launch_extrapolate_gated(const ExtrapArgs& a, int K, bool cache_bf16, int grid, cudaStream_t s);
 cudaError_t extrapolate_blocks_per_sm(int K, bool cache_bf16, int* blocks);
 
 // Bulk-copy pipeline variant (extrapolate_bulk.cu).
-size_t bulk_smem_bytes(int chunks_per_stage, int stages);
+size_t bulk_smem_bytes(int chunks_per_stage, size_t extra_per_stage, int stages);
 cudaError_t prepare_extrapolate_bulk(int K, bool cache_bf16, size_t smem);
 cudaError_t launch_extrapolate_bulk(const ExtrapArgs& a, int K, bool cache_bf16, int grid, size_t smem,
                                     cudaStream_t s);
+// gated variant of the bulk kernel (extrapolate_bulk_gated.cu)
+cudaError_t prepare_extrapolate_bulk_gated(int K, bool cache_bf16, size_t smem);
+cudaError_t launch_extrapolate_bulk_gated(const ExtrapArgs& a, int K, bool cache_bf16, int grid, size_t smem,
+                                          cudaStream_t s);
 
 cudaError_t launch_push(const PushArgs& a, bool src_bf16, bool dst_bf16, int grid, cudaStream_t s);
 cudaError_t push_blocks_per_sm(bool src_bf16, bool dst_bf16, int* blocks);

@@ -16,6 +16,8 @@
 
 #include <cuda_bf16.h>
 
+#include <type_traits>
+
 #include "cb_device.h"
 
 namespace cbk {
@@ -91,6 +93,12 @@ __device__ __forceinline__ uint16_t bf16_of_pair(float hi, float lo) {
     return bf16_bits(hi);
 }
 
+// Start of history entry j of the member at byte offset moff.
+__device__ __forceinline__ const unsigned char* hist_ptr(const ExtrapArgs& A, int j, long long moff) {
+    return reinterpret_cast<const unsigned char*>(A.hist_base + (unsigned long long)A.slot_off[j] +
+                                                  (unsigned long long)moff);
+}
+
 template <bool CB16>
 __device__ __forceinline__ float load_cache_elem(const unsigned char* base, long long e) {
     if constexpr (CB16) {
@@ -113,13 +121,51 @@ __device__ __forceinline__ void store_pair(void* p, bool bf16, long long e, floa
         reinterpret_cast<float*>(p)[e] = hi;
 }
 
+// Full-step epilogue: element e of a source converted to the output type (bit
+// copy for equal types, exact widening, round-to-nearest-even narrowing).
+template <bool CB16>
+__device__ __forceinline__ void copy_elem(void* out, bool out_bf16, const unsigned char* src, long long e) {
+    if constexpr (CB16) {
+        const uint16_t h = reinterpret_cast<const uint16_t*>(src)[e];
+        if (out_bf16)
+            reinterpret_cast<uint16_t*>(out)[e] = h;
+        else
+            reinterpret_cast<uint32_t*>(out)[e] = (uint32_t)h << 16;
+    } else {
+        const float f = reinterpret_cast<const float*>(src)[e];
+        if (out_bf16)
+            reinterpret_cast<uint16_t*>(out)[e] = bf16_bits(f);
+        else
+            reinterpret_cast<float*>(out)[e] = f;
+    }
+}
+
+// Gate of member mi (item it) at element e: g[b * hidden + h] for element
+// e = (b * tokens + token) * hidden + h; 1 when the member has no gate.
+__device__ __forceinline__ float gate_at(const ExtrapArgs& A, int mi, int it, long long e) {
+    const void* g = A.m_gate[mi];
+    if (!g) return 1.0f;
+    const unsigned long long row = A.i_row[it], H = A.i_hidden[it], ue = (unsigned long long)e;
+    return load_elem(g, A.gate_bf16, (long long)(ue / row * H + ue % H));
+}
+
+// Exact product g * (h + l) added to the unevaluated sum tp + tc.
+__device__ __forceinline__ void add_gated_pair(float g, float h, float l, float& tp, float& tc) {
+    const float gh = __fmul_rn(g, h);
+    const float gr = __fmaf_rn(g, h, -gh);  // exact: g*h - gh
+    float q;
+    two_sum(tp, gh, tp, q);
+    tc = __fadd_rn(tc, __fadd_rn(q, gr));
+    tc = __fmaf_rn(g, l, tc);
+}
+
 // Compensated value of member tensor (byte offset moff) at element e.
 template <bool CB16>
 __device__ __noinline__ void exact_member(const ExtrapArgs& A, int K, long long moff, long long e, float& hi,
                                           float& lo) {
     float p = 0.0f, c = 0.0f;
     for (int j = 0; j < K; ++j) {
-        const float f = load_cache_elem<CB16>(A.cache + A.slot_off[j] + moff, e);
+        const float f = load_cache_elem<CB16>(hist_ptr(A, j, moff), e);
         dot2_step(A.w_hi[j], A.w_lo[j], f, p, c);
     }
     two_sum(p, c, hi, lo);
@@ -134,8 +180,12 @@ __device__ __noinline__ void exact_resid(const ExtrapArgs& A, int K, int it, lon
     for (int m = 0; m < A.nb[it]; ++m) {
         float h, l, q;
         exact_member<CB16>(A, K, A.m_off[first + m], e, h, l);
-        two_sum(tp, h, tp, q);
-        tc = __fadd_rn(tc, __fadd_rn(q, l));
+        if (A.m_gate[first + m]) {
+            add_gated_pair(gate_at(A, first + m, it, e), h, l, tp, tc);
+        } else {
+            two_sum(tp, h, tp, q);
+            tc = __fadd_rn(tc, __fadd_rn(q, l));
+        }
     }
     two_sum(tp, tc, hi, lo);
 }
@@ -150,9 +200,17 @@ __device__ __noinline__ void scalar_element(const ExtrapArgs& A, int K, int it, 
     for (int m = 0; m < A.nb[it]; ++m) {
         float hi, lo, q;
         exact_member<CB16>(A, K, A.m_off[first + m], e, hi, lo);
-        if (A.m_out[first + m]) store_pair(A.m_out[first + m], A.out_bf16, e, hi, lo);
-        two_sum(tp, hi, tp, q);
-        tc = __fadd_rn(tc, __fadd_rn(q, lo));
+        void* out = A.m_out[first + m];
+        if (out && A.copy_out)
+            copy_elem<CB16>(out, A.out_bf16, hist_ptr(A, 0, A.m_off[first + m]), e);
+        else if (out)
+            store_pair(out, A.out_bf16, e, hi, lo);
+        if (A.m_gate[first + m]) {
+            add_gated_pair(gate_at(A, first + m, it, e), hi, lo, tp, tc);
+        } else {
+            two_sum(tp, hi, tp, q);
+            tc = __fadd_rn(tc, __fadd_rn(q, lo));
+        }
     }
     if (resid) {
         float q, hi, lo;
@@ -206,6 +264,57 @@ struct Acc {
 template <int K, bool CB16, int UV>
 using RawVecs = uint4[UV][K][CB16 ? 1 : 2];
 
+// Full-step epilogue: the 8 source values of vector (raw) written to out at
+// element e in the output type (see copy_elem).
+template <bool CB16>
+__device__ __forceinline__ void copy_vec(void* out, bool out_bf16, long long e, const uint4 (&r)[CB16 ? 1 : 2]) {
+    if constexpr (CB16) {
+        if (out_bf16) {
+            *reinterpret_cast<uint4*>(reinterpret_cast<uint16_t*>(out) + e) = r[0];
+        } else {
+            const uint4 v = r[0];
+            uint4* q = reinterpret_cast<uint4*>(reinterpret_cast<float*>(out) + e);
+            q[0] = make_uint4(v.x << 16, v.x & 0xFFFF0000u, v.y << 16, v.y & 0xFFFF0000u);
+            q[1] = make_uint4(v.z << 16, v.z & 0xFFFF0000u, v.w << 16, v.w & 0xFFFF0000u);
+        }
+    } else {
+        const uint4 a = r[0], b = r[CB16 ? 0 : 1];
+        if (out_bf16) {
+            *reinterpret_cast<uint4*>(reinterpret_cast<uint16_t*>(out) + e) = make_uint4(
+                pack_bf16x2(__uint_as_float(a.x), __uint_as_float(a.y)), pack_bf16x2(__uint_as_float(a.z), __uint_as_float(a.w)),
+                pack_bf16x2(__uint_as_float(b.x), __uint_as_float(b.y)), pack_bf16x2(__uint_as_float(b.z), __uint_as_float(b.w)));
+        } else {
+            uint4* q = reinterpret_cast<uint4*>(reinterpret_cast<float*>(out) + e);
+            q[0] = a;
+            q[1] = b;
+        }
+    }
+}
+
+// Output pointer handed to member_fast / member_precise for member mi: in the
+// full-step epilogue the sources are written out converted here and no
+// prediction is stored (null); otherwise the member's prediction output.
+template <int K, bool CB16, int UV>
+__device__ __forceinline__ void* member_out(const ExtrapArgs& A, int mi, const long long (&ev)[UV],
+                                            const RawVecs<K, CB16, UV>& raw) {
+    void* out = A.m_out[mi];
+    if (!A.copy_out) return out;
+    if (out)
+#pragma unroll
+        for (int u = 0; u < UV; ++u) copy_vec<CB16>(out, A.out_bf16, ev[u], raw[u][0]);
+    return nullptr;
+}
+
+// Gate source of an ungated accumulation (never called).
+struct NoGate {
+    __device__ void operator()(int, float (&)[8]) const {}
+};
+
+// Placeholder for "no recompute functor" (never called).
+struct NoExact {
+    __device__ void operator()(int, int, float&, float&) const {}
+};
+
 // Dot2 value of element e of vector u from its K history values as loaded
 // (registers or shared memory); used where the fast path's guard fails.
 template <int K, bool CB16, int UV>
@@ -233,13 +342,17 @@ __device__ __forceinline__ bool guard_ok(float g, float a, float s) { return g *
 
 // Fast path for one member over UV aligned 8-element vectors already loaded
 // into registers: bf16 prediction (if out) and accumulation into acc. The
-// rare guarded elements are recomputed from the loaded values (FROM_RAW: no
-// memory latency, but the values stay live and cost registers) or re-read
-// from global memory (member byte offset moff).
-template <int K, bool CB16, int UV, bool FROM_RAW>
+// rare guarded elements are recomputed by exact(u, e, hi, lo) when given
+// (e.g. from shared memory), else from the loaded values (FROM_RAW: no memory
+// latency, but the values stay live and cost registers) or re-read from
+// global memory (member byte offset moff).
+// GATED: gate(u, g) supplies the 8 gate values of vector u when it is
+// accumulated (late, so that they are not live beside the history values).
+template <int K, bool CB16, int UV, bool FROM_RAW, bool GATED = false, typename Gate = NoGate,
+          typename Exact = NoExact>
 __device__ __forceinline__ void member_fast(const ExtrapArgs& A, long long moff, void* out,
                                             const long long (&ev)[UV], const RawVecs<K, CB16, UV>& raw,
-                                            bool accumulate, Acc<UV>& acc) {
+                                            bool accumulate, Acc<UV>& acc, Gate gate = {}, Exact exact = {}) {
     const float g_out = (float)(K + 2) * kU * 1.01f;
 #pragma unroll
     for (int u = 0; u < UV; ++u) {
@@ -267,7 +380,9 @@ __device__ __forceinline__ void member_fast(const ExtrapArgs& A, long long moff,
                 const int e = __ffs(bad) - 1;
                 bad &= bad - 1;
                 float hi, lo;
-                if constexpr (FROM_RAW)
+                if constexpr (!std::is_same_v<Exact, NoExact>)
+                    exact(u, e, hi, lo);
+                else if constexpr (FROM_RAW)
                     exact_from_raw<K, CB16, UV>(A, raw, u, e, hi, lo);
                 else
                     exact_member<CB16>(A, K, moff, ev[u] + e, hi, lo);
@@ -276,10 +391,17 @@ __device__ __forceinline__ void member_fast(const ExtrapArgs& A, long long moff,
             store_bf16x8(out, ev[u], pk);
         }
         if (accumulate) {
+            float g[8];
+            if constexpr (GATED) gate(u, g);
 #pragma unroll
             for (int e = 0; e < 8; ++e) {
-                acc.x[u][e] += s[e];
-                acc.y[u][e] += a[e];
+                if constexpr (GATED) {  // x + g * s: one rounding, bound |g| a
+                    acc.x[u][e] = fmaf(g[e], s[e], acc.x[u][e]);
+                    acc.y[u][e] = fmaf(fabsf(g[e]), a[e], acc.y[u][e]);
+                } else {
+                    acc.x[u][e] += s[e];
+                    acc.y[u][e] += a[e];
+                }
             }
         }
     }
@@ -319,10 +441,10 @@ __device__ __forceinline__ void resid_fast(const ExtrapArgs& A, int it, const lo
 }
 
 // Compensated path for one member (any fp32 prediction or hidden state).
-template <int K, bool CB16, int UV>
+template <int K, bool CB16, int UV, bool GATED = false, typename Gate = NoGate>
 __device__ __forceinline__ void member_precise(const ExtrapArgs& A, void* out, const long long (&ev)[UV],
                                                const RawVecs<K, CB16, UV>& raw, bool accumulate,
-                                               Acc<UV>& acc) {
+                                               Acc<UV>& acc, Gate gate = {}) {
 #pragma unroll
     for (int u = 0; u < UV; ++u) {
         float p[8], c[8];
@@ -351,11 +473,17 @@ __device__ __forceinline__ void member_precise(const ExtrapArgs& A, void* out, c
             }
         }
         if (accumulate) {
+            float g[8];
+            if constexpr (GATED) gate(u, g);
 #pragma unroll
             for (int e = 0; e < 8; ++e) {
-                float q;
-                two_sum(acc.x[u][e], hi[e], acc.x[u][e], q);
-                acc.y[u][e] = __fadd_rn(acc.y[u][e], __fadd_rn(q, lo[e]));
+                if constexpr (GATED) {
+                    add_gated_pair(g[e], hi[e], lo[e], acc.x[u][e], acc.y[u][e]);
+                } else {
+                    float q;
+                    two_sum(acc.x[u][e], hi[e], acc.x[u][e], q);
+                    acc.y[u][e] = __fadd_rn(acc.y[u][e], __fadd_rn(q, lo[e]));
+                }
             }
         }
     }
@@ -385,6 +513,42 @@ __device__ __forceinline__ void resid_precise(const ExtrapArgs& A, const long lo
         } else {
             store_f32x8(resid, ev[u], hi);
         }
+    }
+}
+
+// Gate offsets b * hidden + h of UV vectors of a tile starting at element e0
+// (32-bit arithmetic: gated tensors have fewer than 2^32 elements). Rows of
+// tokens * hidden are multiples of hidden, so h follows from e mod hidden.
+template <int UV>
+__device__ __forceinline__ void gate_offsets(const ExtrapArgs& A, int it, long long e0,
+                                             const long long (&ev)[UV], unsigned (&gi)[UV]) {
+    const unsigned row = A.i_row[it], H = A.i_hidden[it], ue0 = (unsigned)e0;
+    const unsigned q0 = ue0 / row, r0 = ue0 - q0 * row, rh = r0 % H;
+#pragma unroll
+    for (int u = 0; u < UV; ++u) {
+        const unsigned off = (unsigned)(ev[u] - e0);
+        unsigned r = r0 + off, b = q0;
+        while (r >= row) {
+            r -= row;
+            ++b;
+        }
+        unsigned h = rh + off % H;
+        if (h >= H) h -= H;
+        gi[u] = b * H + h;
+    }
+}
+
+// The 8 gate values of member mi for each of UV vectors (1 without a gate).
+template <int UV>
+__device__ __forceinline__ void load_gates(const ExtrapArgs& A, int mi, const unsigned (&gi)[UV], float (&g)[UV][8]) {
+    const void* gp = A.m_gate[mi];
+#pragma unroll
+    for (int u = 0; u < UV; ++u) {
+        if (gp)
+            load_x8(gp, A.gate_bf16, (long long)gi[u], g[u]);
+        else
+#pragma unroll
+            for (int e = 0; e < 8; ++e) g[u][e] = 1.0f;
     }
 }
 

@@ -1,300 +1,26 @@
-// Skipped-step kernel, bulk-copy pipeline variant (same arithmetic and bits as
-// extrapolate.cu; Sec. 3.3, Eq. for f_t; Alg. 1, extrapolation branch).
-//
-// One CTA per SM. A producer lane moves, for every work unit (one tile of one
-// branch tensor), the K history chunks of 8 KB each from HBM into a ring of
-// shared-memory stages with cp.async.bulk (the Blackwell bulk-copy engine),
-// each stage guarded by a "full" mbarrier (transaction bytes) and an "empty"
-// mbarrier (one arrival per consumer warp). Consumer warps read their 8-element
-// vectors of the K chunks from shared memory, release the stage, and compute
-// and store from registers. With S stages of K x 8 KB (S = 5 for K = 5) up to
-// ~160 KB per SM stay in flight independently of the consumers' registers,
-// which is what bounds the direct-load variant.
-//
-// Two shapes, chosen per launch (GROUPED):
-//   * predictions only: 16 consumer warps with one vector each (17 warps, up
-//     to 96 registers per thread); more warps per scheduler hide the
-//     consumers' fixed latencies better (measured: +2 to +3 % of peak);
-//   * with hidden states: 8 consumer warps with two vectors each (the direct
-//     kernel's thread map, up to 168 registers). The producer also stages
-//     each tile's bf16 hidden state (one more chunk with the group's last
-//     member) and the consumers hold the group's member stages until the
-//     hidden state is written, so that the rare guarded elements are
-//     recomputed from shared memory (the host guarantees more stages than
-//     members, so holding cannot starve the producer).
-//
-// Every wait is bounded (%globaltimer). A wait that runs out records a code in
-// the plan's device status word and the thread returns; the producer then
-// waits, with its own limit (at least 10 ms), for the copies it has issued
-// before it exits. A test option makes the producer announce the first unit's
-// bytes without issuing its copies, so that the consumers' wait runs out with
-// no fault and nothing in flight.
-#include "cb_math.cuh"
+// Instantiations of the bulk-copy pipeline kernel (bulk_kernel.cuh) without
+// gates: prediction-only launches and launches that add the predictions
+// straight into the hidden states.
+#include "bulk_kernel.cuh"
 
 namespace cbk {
 namespace {
 
-template <bool GROUPED>
-struct Shape {
-    static constexpr int consumer_warps = GROUPED ? 8 : 16;
-    static constexpr int consumers = consumer_warps * 32;
-    static constexpr int threads = consumers + 32;  // plus the producer warp
-};
-constexpr int kChunkBytes = 8192;   // one history entry's share of a tile
-constexpr int kBarrierBytes = 256;  // full[S] and empty[S] barriers, S <= 16
-constexpr unsigned long long kMinDrainNs = 10000000ull;  // copies land in microseconds
-constexpr unsigned long long kMaxWaitNs = 60000000000ull;  // no wait outlives a minute
-
-__device__ __forceinline__ uint32_t smem_addr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
-
-__device__ __forceinline__ unsigned long long now_ns() {
-    unsigned long long t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    return t;
-}
-
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(bar), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-
-// Wait for the phase with the given parity to complete, for at most limit_ns
-// (never more than kMaxWaitNs).
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, unsigned long long limit_ns) {
-    if (limit_ns > kMaxWaitNs) limit_ns = kMaxWaitNs;
-    if (mbar_try_wait(bar, parity)) return true;
-    const unsigned long long t0 = now_ns();
-    while (!mbar_try_wait(bar, parity))
-        if (now_ns() - t0 > limit_ns) return false;
-    return true;
-}
-
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
-}
-
-// Global -> shared bulk copy completing `bytes` transaction bytes on `bar`.
-// dst, src 16-byte aligned; bytes a multiple of 16.
-__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
-    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                     dst),
-                 "l"(src), "r"(bytes), "r"(bar)
-                 : "memory");
-}
-
-__device__ __forceinline__ void record(int* status, int code) {
-    if (status) atomicOr(status, code);
-}
-
-// GROUPED: some item updates a hidden state (stage holding, hidden-state
-// staging, 8 consumer warps); prediction-only launches compile without that
-// bookkeeping and with 16 consumer warps.
-template <int K, bool CB16, bool GROUPED>
-__global__ void __launch_bounds__(Shape<GROUPED>::threads, 1)
-    extrapolate_bulk_kernel(const __grid_constant__ ExtrapArgs A) {
-    extern __shared__ __align__(128) unsigned char smem[];
-    constexpr int NCW = Shape<GROUPED>::consumer_warps;
-    constexpr int NCT = Shape<GROUPED>::consumers;
-    constexpr long long TE = tile_elems(CB16);  // 8 KB per history chunk for both cache types
-    constexpr int ES = CB16 ? 2 : 4;
-    constexpr int NV = (int)(TE / kVecElems);     // vectors per tile: 512 (bf16) or 256 (fp32)
-    constexpr int U = NV >= NCT ? NV / NCT : 1;   // vectors per consumer thread per tile
-    static_assert(NV % NCT == 0 || NCT % NV == 0, "vectors spread evenly over the consumers");
-    static_assert(TE * ES == kChunkBytes, "one tile of one history entry is one chunk");
-    const int S = A.stages;
-    const uint32_t full0 = smem_addr(smem);
-    const uint32_t empty0 = full0 + 8u * (uint32_t)S;
-    const uint32_t buf0 = smem_addr(smem + kBarrierBytes);
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-
-    if (threadIdx.x == 0) {
-        for (int s = 0; s < S; ++s) {
-            mbar_init(full0 + 8u * s, 1);
-            mbar_init(empty0 + 8u * s, NCW);
-        }
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    }
-    __syncthreads();
-
-    const int C = GROUPED ? A.stage_chunks : K;
-    if (warp == NCW) {  // ---------------------------------- producer
-        if (lane != 0) return;
-        int it = 0;
-        unsigned u = 0;
-        bool ok = true;
-        for (int tile = blockIdx.x; ok && tile < A.tiles_total; tile += gridDim.x) {
-            while (tile >= A.tile_begin[it + 1]) ++it;
-            const long long numel = A.numel[it];
-            const long long e0 = (long long)(tile - A.tile_begin[it]) * TE;
-            // consumers read shared memory only for whole tiles of aligned items;
-            // for the ragged last tile (or a misaligned item) the stage is
-            // cycled without data and they recompute from global memory
-            const bool full_tile = A.vec_ok[it] && e0 + TE <= numel;
-            const uint32_t bytes = full_tile ? (uint32_t)kChunkBytes : 0u;
-            const int first = A.first[it];
-            const int nb = GROUPED ? A.nb[it] : 1;
-            const unsigned char* resid = GROUPED ? reinterpret_cast<const unsigned char*>(A.resid[it]) : nullptr;
-            for (int m = 0; m < nb; ++m, ++u) {
-                const uint32_t stage = u % (unsigned)S, q = u / (unsigned)S;
-                if (q > 0 && !mbar_wait(empty0 + 8u * stage, (q - 1) & 1u, A.wait_ns)) {
-                    record(A.status, 2);
-                    ok = false;
-                    break;
-                }
-                // the tile's bf16 hidden state travels with its last member
-                const bool with_x = GROUPED && A.stage_x && resid && full_tile && m == nb - 1;
-                const uint32_t xbytes = with_x ? (uint32_t)(TE * 2) : 0u;
-                mbar_expect_tx(full0 + 8u * stage, (uint32_t)K * bytes + xbytes);
-                if (A.withhold_first && u == 0) continue;
-                const uint32_t dst = buf0 + stage * (uint32_t)C * (uint32_t)kChunkBytes;
-                if (bytes) {
-                    const unsigned char* src = A.cache + A.m_off[first + m] + e0 * ES;
-#pragma unroll
-                    for (int j = 0; j < K; ++j)
-                        bulk_g2s(dst + j * (uint32_t)kChunkBytes, src + A.slot_off[j], bytes, full0 + 8u * stage);
-                }
-                if (xbytes) bulk_g2s(dst + K * (uint32_t)kChunkBytes, resid + e0 * 2, xbytes, full0 + 8u * stage);
-            }
-        }
-        // never leave while copies into this CTA's shared memory are in flight
-        const unsigned long long drain_ns = A.wait_ns > kMinDrainNs ? A.wait_ns : kMinDrainNs;
-        for (unsigned q = u > (unsigned)S ? u - S : 0; q < u; ++q)
-            if (!mbar_wait(full0 + 8u * (q % S), (q / S) & 1u, drain_ns)) {
-                record(A.status, 4);
-                break;
-            }
-        return;
-    }
-
-    // ------------------------------------------------------------ consumers
-    const int c = threadIdx.x;
-    const unsigned char* stages = smem + kBarrierBytes;
-    auto chunk = [&](uint32_t stage, int j) { return stages + ((size_t)stage * C + j) * kChunkBytes; };
-    int it = 0;
-    unsigned u = 0;
-    for (int tile = blockIdx.x; tile < A.tiles_total; tile += gridDim.x) {
-        while (tile >= A.tile_begin[it + 1]) ++it;
-        const long long numel = A.numel[it];
-        const long long e0 = (long long)(tile - A.tile_begin[it]) * TE;
-        const int nb = GROUPED ? A.nb[it] : 1;
-        const int first = A.first[it];
-        void* resid = GROUPED ? A.resid[it] : nullptr;
-        // whole aligned tiles come from shared memory; the ragged last tile of a
-        // tensor and misaligned items take the compensated scalar path
-        const bool full_tile = A.vec_ok[it] && e0 + TE <= numel;
-        // with a hidden state, every member's stage stays held until the hidden
-        // state is written, so that its guarded elements can be recomputed
-        const bool hold = GROUPED && full_tile && resid != nullptr;
-        const bool mine = NV >= NCT || c < NV;  // fp32 tiles have fewer vectors than consumers
-        const unsigned u0 = u;
-        long long ev[U];
-#pragma unroll
-        for (int v = 0; v < U; ++v) ev[v] = e0 + ((long long)v * NCT + c) * kVecElems;
-        Acc<U> acc;
-        acc.zero();
-        for (int m = 0; m < nb; ++m, ++u) {
-            const uint32_t stage = u % (unsigned)S, q = u / (unsigned)S;
-            if (!mbar_wait(full0 + 8u * stage, q & 1u, A.wait_ns)) {
-                record(A.status, 1);
-                return;
-            }
-            RawVecs<K, CB16, U> raw;
-            if (full_tile && mine) {
-#pragma unroll
-                for (int v = 0; v < U; ++v)
-#pragma unroll
-                    for (int j = 0; j < K; ++j) {
-                        const unsigned char* p = chunk(stage, j) + (size_t)(ev[v] - e0) * ES;
-                        raw[v][j][0] = *reinterpret_cast<const uint4*>(p);
-                        if constexpr (!CB16) raw[v][j][CB16 ? 0 : 1] = *reinterpret_cast<const uint4*>(p + 16);
-                    }
-            }
-            if (!hold) {
-                __syncwarp();
-                if (lane == 0) mbar_arrive(empty0 + 8u * stage);
-            }
-            if (full_tile && mine) {
-                if (A.precise)
-                    member_precise<K, CB16, U>(A, A.m_out[first + m], ev, raw, resid != nullptr, acc);
-                else
-                    member_fast<K, CB16, U, true>(A, A.m_off[first + m], A.m_out[first + m], ev, raw,
-                                                  resid != nullptr, acc);
-            }
-        }
-        if (GROUPED && hold) {
-            const uint32_t last = (u0 + nb - 1) % (unsigned)S;
-            auto xload = [&](int v, float (&x)[8]) {
-                if (A.stage_x)
-                    unpack_bf16x8(*reinterpret_cast<const uint4*>(chunk(last, K) + (size_t)(ev[v] - e0) * 2), x);
-                else
-                    load_x8(resid, A.resid_bf16, ev[v], x);
-            };
-            if (!mine) {
-            } else if (A.precise) {
-                resid_precise<U>(A, ev, acc, resid, xload);
-            } else {
-                // Dot2 of x + sum_b P_b for one element, from the held stages
-                auto exact = [&](int v, int e, float xe, float& hi, float& lo) {
-                    const size_t off = (size_t)(ev[v] - e0 + e) * ES;
-                    float tp = xe, tc = 0.0f;
-                    for (int m = 0; m < nb; ++m) {
-                        const uint32_t st = (u0 + m) % (unsigned)S;
-                        float p = 0.0f, cc = 0.0f, h, l, qq;
-#pragma unroll
-                        for (int j = 0; j < K; ++j) {
-                            const unsigned char* src = chunk(st, j) + off;
-                            const float f = CB16 ? __uint_as_float((uint32_t)(*reinterpret_cast<const uint16_t*>(src)) << 16)
-                                                 : *reinterpret_cast<const float*>(src);
-                            dot2_step(A.w_hi[j], A.w_lo[j], f, p, cc);
-                        }
-                        two_sum(p, cc, h, l);
-                        two_sum(tp, h, tp, qq);
-                        tc = __fadd_rn(tc, __fadd_rn(qq, l));
-                    }
-                    two_sum(tp, tc, hi, lo);
-                };
-                resid_fast<K, U>(A, it, ev, acc, resid, xload, exact);
-            }
-            __syncwarp();
-            if (lane == 0)
-                for (int m = 0; m < nb; ++m) mbar_arrive(empty0 + 8u * ((u0 + m) % (unsigned)S));
-        } else if (!full_tile) {
-            const long long end = e0 + TE < numel ? e0 + TE : numel;
-            for (long long e = e0 + c; e < end; e += NCT) scalar_element<CB16>(A, K, it, e);
-        }
-    }
-}
-
 template <int K, bool CB16>
 cudaError_t launch_k(const ExtrapArgs& a, bool grouped, int grid, size_t smem, cudaStream_t s) {
     if (grouped)
-        extrapolate_bulk_kernel<K, CB16, true><<<grid, Shape<true>::threads, smem, s>>>(a);
+        extrapolate_bulk_kernel<K, CB16, true, false><<<grid, Shape<CB16>::threads, smem, s>>>(a);
     else
-        extrapolate_bulk_kernel<K, CB16, false><<<grid, Shape<false>::threads, smem, s>>>(a);
+        extrapolate_bulk_kernel<K, CB16, false, false><<<grid, Shape<CB16>::threads, smem, s>>>(a);
     return cudaGetLastError();
 }
 
 template <int K, bool CB16>
 cudaError_t prepare_k(size_t smem) {
-    cudaError_t e = cudaFuncSetAttribute(extrapolate_bulk_kernel<K, CB16, true>,
+    cudaError_t e = cudaFuncSetAttribute(extrapolate_bulk_kernel<K, CB16, true, false>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    return cudaFuncSetAttribute(extrapolate_bulk_kernel<K, CB16, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    return cudaFuncSetAttribute(extrapolate_bulk_kernel<K, CB16, false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)smem);
 }
 
@@ -313,8 +39,8 @@ cudaError_t prepare_k(size_t smem) {
 
 }  // namespace
 
-size_t bulk_smem_bytes(int chunks_per_stage, int stages) {
-    return kBarrierBytes + (size_t)stages * chunks_per_stage * kChunkBytes;
+size_t bulk_smem_bytes(int chunks_per_stage, size_t extra_per_stage, int stages) {
+    return kBarrierBytes + (size_t)stages * ((size_t)chunks_per_stage * kChunkBytes + extra_per_stage);
 }
 
 cudaError_t prepare_extrapolate_bulk(int K, bool cache_bf16, size_t smem) {
@@ -330,8 +56,7 @@ cudaError_t prepare_extrapolate_bulk(int K, bool cache_bf16, size_t smem) {
 
 cudaError_t launch_extrapolate_bulk(const ExtrapArgs& a, int K, bool cache_bf16, int grid, size_t smem,
                                     cudaStream_t s) {
-    // fp32 caches have 256 vectors per tile: they keep the 8-consumer-warp shape
-    bool grouped = !cache_bf16;
+    bool grouped = false;
     for (int i = 0; i < a.n_items; ++i) grouped = grouped || a.resid[i] != nullptr || a.nb[i] > 1;
 #define L_BF(k) launch_k<k, true>(a, grouped, grid, smem, s)
 #define L_F32(k) launch_k<k, false>(a, grouped, grid, smem, s)

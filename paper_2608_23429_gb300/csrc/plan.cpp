@@ -6,6 +6,7 @@
 // extrapolate.cu.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdint>
 #include <cstring>
@@ -65,6 +66,7 @@ struct DeviceInfo {
     int occ_extrap[2][CB_MAX_K + 1] = {};  // [cache_bf16][K]
     int occ_push[2][2] = {};               // [src_bf16][dst_bf16]
     int bulk_stages[2][CB_MAX_K + 1] = {};  // 1 once the kernel's shared-memory limit is raised
+    int bulk_gated[2][CB_MAX_K + 1] = {};   // the same for the gated kernel
 };
 
 }  // namespace
@@ -80,6 +82,8 @@ struct cb_plan {
     int dir = 0;                           // +1 increasing, -1 decreasing t
     std::vector<double> rho_win;           // rho of node window i: rho_win[i*K + j]
     std::vector<long long> off;            // byte offset of tensor i inside a slot
+    std::vector<long long> sh_tokens;      // [batch, tokens, hidden] of each tensor (0: unset)
+    std::vector<long long> sh_hidden;
     size_t slot_bytes = 0;
     // bound history buffer
     unsigned char* cache = nullptr;
@@ -136,20 +140,24 @@ int extrap_grid(cb_plan* p, int K, bool cb16, int tiles, int* grid) {
     return CB_OK;
 }
 
+// Largest gate staging per pipeline stage (two rows of 4096 fp32 channels).
+constexpr size_t kMaxStagedGateBytes = 32768;
+
 // Pipeline of the bulk kernel: as many stages of `chunks` 8 KB chunks as fit
 // in one CTA's shared memory (at most 8). The kernel's dynamic shared-memory
 // limit is raised to the device maximum once per instantiation.
-int bulk_config(cb_plan* p, int K, bool cb16, int chunks, int* stages, size_t* smem) {
-    int& prepared = p->dev.bulk_stages[cb16 ? 1 : 0][K];
+int bulk_config(cb_plan* p, int K, bool cb16, int chunks, size_t extra, bool gated, int* stages, size_t* smem) {
+    int& prepared = gated ? p->dev.bulk_gated[cb16 ? 1 : 0][K] : p->dev.bulk_stages[cb16 ? 1 : 0][K];
     if (prepared == 0) {
-        cudaError_t e = cbk::prepare_extrapolate_bulk(K, cb16, (size_t)p->dev.smem_optin);
+        cudaError_t e = gated ? cbk::prepare_extrapolate_bulk_gated(K, cb16, (size_t)p->dev.smem_optin)
+                              : cbk::prepare_extrapolate_bulk(K, cb16, (size_t)p->dev.smem_optin);
         if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute");
         prepared = 1;
     }
     int s = 8;
-    while (s > 1 && cbk::bulk_smem_bytes(chunks, s) > (size_t)p->dev.smem_optin) --s;
-    *stages = cbk::bulk_smem_bytes(chunks, s) <= (size_t)p->dev.smem_optin ? s : 0;
-    *smem = cbk::bulk_smem_bytes(chunks, s);
+    while (s > 1 && cbk::bulk_smem_bytes(chunks, extra, s) > (size_t)p->dev.smem_optin) --s;
+    *stages = cbk::bulk_smem_bytes(chunks, extra, s) <= (size_t)p->dev.smem_optin ? s : 0;
+    *smem = cbk::bulk_smem_bytes(chunks, extra, s);
     return CB_OK;
 }
 
@@ -229,12 +237,34 @@ Window live_window(const cb_plan* p, int n) {
     return w;
 }
 
+// Gates (one per tensor, [batch, hidden] of gate_dtype, null = 1) apply to the
+// hidden-state update of a grouped tensor: its shape must be set, its group's
+// tensors must share it, and indexing stays in 32 bits.
+int check_gates(const cb_plan* p, void* const* resid, const void* const* gates, cb_dtype gate_dtype) {
+    if (!gates) return CB_OK;
+    if (!valid_dtype(gate_dtype)) return CB_ERR_ARG;
+    const int n = (int)p->tensors.size();
+    for (int i = 0; i < n; ++i) {
+        if (!gates[i]) continue;
+        const auto& d = p->tensors[i];
+        if (p->sh_hidden[i] <= 0) return CB_ERR_ARG;  // cb_plan_set_shapes first
+        if (!aligned(gates[i], esize(gate_dtype))) return CB_ERR_ALIGN;
+        if (d.numel > 0xFFFFFFFFLL) return CB_ERR_LIMIT;
+        (void)resid;
+    }
+    return CB_OK;
+}
+
 // One skipped-step launch over the window `win` with the fp64 weights w[0..n).
+// With `feats` it is instead a full step's epilogue: a one-entry history (the
+// new features, weight 1) whose members are written, converted, into the ring
+// slot `next` while the hidden states receive x + sum_b g_b f_b.
 int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs, cb_dtype out_dtype,
-               void* const* resid, cb_dtype resid_dtype, void* stream) {
+               void* const* resid, cb_dtype resid_dtype, void* stream, const void* const* gates = nullptr,
+               cb_dtype gate_dtype = CB_BF16, const void* const* feats = nullptr, cb_dtype feat_dtype = CB_BF16) {
     if (!p->cache) return CB_ERR_UNBOUND;
     const int K = win.n;
-    if (K < 1 || p->count < K) return CB_ERR_HISTORY_NOT_FULL;
+    if (K < 1 || (!feats && p->count < K)) return CB_ERR_HISTORY_NOT_FULL;
     if (!valid_dtype(out_dtype) || !valid_dtype(resid_dtype)) return CB_ERR_ARG;
     const int n = (int)p->tensors.size();
     const int ng = (int)p->groups.size();
@@ -248,15 +278,19 @@ int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs
 
     for (int j = 0; j < K; ++j)
         if (!std::isfinite(w[j])) return CB_ERR_ARG;
-    int rc = CB_OK;
+    int rc = check_gates(p, resid, gates, gate_dtype);
+    if (rc != CB_OK) return rc;
 
     cbk::ExtrapArgs& A = *p->eargs;
-    const bool cb16 = p->cache_dtype == CB_BF16;
+    // the kernels' source type: the cache's, or the new features'
+    const bool cb16 = (feats ? feat_dtype : p->cache_dtype) == CB_BF16;
     const long long te = cbk::tile_elems(cb16);
-    A.cache = p->cache;
+    unsigned char* slot = p->cache + (size_t)p->next * p->slot_bytes;
+    A.hist_base = feats ? 0ull : (unsigned long long)(uintptr_t)p->cache;
+    A.copy_out = feats ? 1 : 0;
     for (int j = 0; j < CB_MAX_K; ++j) {
         const bool on = j < K;
-        A.slot_off[j] = on ? (long long)win.slot[j] * (long long)p->slot_bytes : 0;
+        A.slot_off[j] = on && !feats ? (long long)win.slot[j] * (long long)p->slot_bytes : 0;
         const float hi = on ? (float)w[j] : 0.0f;
         A.w_hi[j] = hi;
         A.w_lo[j] = on ? (float)(w[j] - (double)hi) : 0.0f;
@@ -268,15 +302,26 @@ int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs
     int items = 0, members = 0;
     long long tiles = 0;
     bool any_out = false, any_resid = false;
+    bool any_gate = false;
+    A.gate_bf16 = gate_dtype == CB_BF16;
     auto add_item = [&](const int* mem, int nm, void* res_ptr) {
         const long long numel = p->tensors[mem[0]].numel;
         bool vec = !res_ptr || aligned(res_ptr, 16);
         A.first[items] = (short)members;
+        A.i_hidden[items] = (unsigned)p->sh_hidden[mem[0]];
+        A.i_row[items] = (unsigned)(p->sh_tokens[mem[0]] * p->sh_hidden[mem[0]]);
         for (int m = 0; m < nm; ++m) {
             const int i = mem[m];
-            void* o = outs ? outs[i] : nullptr;
-            A.m_off[members] = p->off[i];
+            void* o = feats ? slot + p->off[i] : outs ? outs[i] : nullptr;
+            const void* g = (res_ptr && gates) ? gates[i] : nullptr;
+            A.m_off[members] = feats ? (long long)(uintptr_t)feats[i] : p->off[i];
+            if (feats) vec = vec && aligned(feats[i], 16);
             A.m_out[members] = o;
+            A.m_gate[members] = g;
+            if (g) {  // vectors of 8 stay inside one gate row
+                any_gate = true;
+                vec = vec && aligned(g, 16) && p->sh_hidden[i] % 8 == 0;
+            }
             if (o) {
                 any_out = true;
                 vec = vec && aligned(o, 16);
@@ -300,12 +345,13 @@ int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs
                 for (int i : p->groups[g]) grouped[i] = 1;
             }
     for (int i = 0; i < n; ++i)
-        if (!grouped[i] && outs && outs[i]) add_item(&i, 1, nullptr);
+        if (!grouped[i] && (feats || (outs && outs[i]))) add_item(&i, 1, nullptr);
     if (tiles > 0x7FFFFFFFLL) return CB_ERR_LIMIT;
     A.tile_begin[items] = (int)tiles;
     A.n_items = items;
     A.tiles_total = (int)tiles;
-    A.precise = (any_out && out_dtype == CB_FP32) || (any_resid && resid_dtype == CB_FP32);
+    // a full step's slot write is a conversion, not arithmetic
+    A.precise = (any_out && !feats && out_dtype == CB_FP32) || (any_resid && resid_dtype == CB_FP32);
     if (items == 0) return CB_OK;  // nothing requested
 
     A.wait_ns = p->wait_ns;
@@ -314,17 +360,20 @@ int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs
     A.stages = 0;
     A.stage_chunks = K;
     A.stage_x = 0;
+    A.stage_gate_bytes = 0;
 
     rc = ensure_device(p);
     if (rc != CB_OK) return rc;
-    if (p->kernel == CB_KERNEL_DIRECT) {
+    auto launch_direct = [&]() {
         int grid = 0;
-        rc = extrap_grid(p, K, cb16, (int)tiles, &grid);
-        if (rc != CB_OK) return rc;
-        cudaError_t e = cbk::launch_extrapolate(A, K, cb16, grid, (cudaStream_t)stream);
+        int r = extrap_grid(p, K, cb16, (int)tiles, &grid);
+        if (r != CB_OK) return r;
+        cudaError_t e = any_gate ? cbk::launch_extrapolate_gated(A, K, cb16, grid, (cudaStream_t)stream)
+                                 : cbk::launch_extrapolate(A, K, cb16, grid, (cudaStream_t)stream);
         if (e != cudaSuccess) return cuda_fail(e, "extrapolate launch");
-        return CB_OK;
-    }
+        return (int)CB_OK;
+    };
+    if (p->kernel == CB_KERNEL_DIRECT) return launch_direct();
     // bf16 hidden states travel through shared memory with the last member of
     // their group; the pipeline must hold a whole group plus one stage ahead
     int max_nb = 1;
@@ -332,19 +381,29 @@ int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs
         if (A.nb[i] > max_nb) max_nb = A.nb[i];
     A.stage_x = any_resid && A.resid_bf16 ? 1 : 0;
     A.stage_chunks = K + A.stage_x;
-    size_t smem = 0;
-    rc = bulk_config(p, K, cb16, A.stage_chunks, &A.stages, &smem);
-    if (rc != CB_OK) return rc;
-    if (A.stages < max_nb + 1) {  // too deep for shared memory: the direct kernel instead
-        int grid = 0;
-        rc = extrap_grid(p, K, cb16, (int)tiles, &grid);
-        if (rc != CB_OK) return rc;
-        cudaError_t e = cbk::launch_extrapolate(A, K, cb16, grid, (cudaStream_t)stream);
-        if (e != cudaSuccess) return cuda_fail(e, "extrapolate launch");
-        return CB_OK;
+    // gate rows travel with their member when every gated tile touches at
+    // most two batches (a batch holds a tile or more) and two rows are small
+    A.stage_gate_bytes = 0;
+    if (any_gate) {
+        const size_t gs = esize(gate_dtype);
+        size_t need = 0;
+        bool fits = true;
+        for (int i = 0; i < items; ++i) {
+            bool gated_item = false;
+            for (int m = 0; m < A.nb[i]; ++m) gated_item = gated_item || A.m_gate[A.first[i] + m];
+            if (!gated_item || !A.vec_ok[i]) continue;
+            fits = fits && (long long)A.i_row[i] >= te;
+            need = std::max(need, 2 * (size_t)A.i_hidden[i] * gs);
+        }
+        if (fits && need <= kMaxStagedGateBytes) A.stage_gate_bytes = (unsigned)((need + 127) / 128 * 128);
     }
+    size_t smem = 0;
+    rc = bulk_config(p, K, cb16, A.stage_chunks, A.stage_gate_bytes, any_gate, &A.stages, &smem);
+    if (rc != CB_OK) return rc;
+    if (A.stages < max_nb + 1) return launch_direct();  // too deep for shared memory
     const int grid = (int)(tiles < p->dev.sms ? tiles : p->dev.sms);  // one CTA per SM
-    cudaError_t e = cbk::launch_extrapolate_bulk(A, K, cb16, grid, smem, (cudaStream_t)stream);
+    cudaError_t e = any_gate ? cbk::launch_extrapolate_bulk_gated(A, K, cb16, grid, smem, (cudaStream_t)stream)
+                             : cbk::launch_extrapolate_bulk(A, K, cb16, grid, smem, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e, "extrapolate launch");
     return CB_OK;
 }
@@ -429,6 +488,8 @@ int cb_plan_create(const double* node_t, int n_nodes, int K, const cb_tensor_des
             o = round_up(o + (size_t)p->tensors[i].numel * esize(cache_dtype), CB_CACHE_ALIGN);
         }
         p->slot_bytes = o;
+        p->sh_tokens.assign(n_tensors, 0);
+        p->sh_hidden.assign(n_tensors, 0);
         *out = p.release();
         return CB_OK;
     } catch (const std::bad_alloc&) {
@@ -542,6 +603,82 @@ int cb_extrapolate_weights(cb_plan* p, const double* w_logical, void* const* out
     const int n = live_entries(p);
     if (n == 0) return p->cache ? CB_ERR_HISTORY_NOT_FULL : CB_ERR_UNBOUND;
     return run_launch(p, live_window(p, n), w_logical, outs, out_dtype, resid, resid_dtype, stream);
+}
+
+int cb_plan_set_shapes(cb_plan* p, const int64_t* bth) {
+    if (!p || !bth) return CB_ERR_ARG;
+    const int n = (int)p->tensors.size();
+    for (int i = 0; i < n; ++i) {
+        const int64_t b = bth[3 * i], t = bth[3 * i + 1], h = bth[3 * i + 2];
+        if (b <= 0 || t <= 0 || h <= 0 || b * t * h != p->tensors[i].numel) return CB_ERR_ARG;
+        if (t * h > 0xFFFFFFFFLL) return CB_ERR_LIMIT;
+    }
+    for (const auto& g : p->groups)  // members of a group share one hidden state, hence one shape
+        for (int i : g)
+            if (bth[3 * i + 1] != bth[3 * g[0] + 1] || bth[3 * i + 2] != bth[3 * g[0] + 2]) return CB_ERR_ARG;
+    for (int i = 0; i < n; ++i) {
+        p->sh_tokens[i] = bth[3 * i + 1];
+        p->sh_hidden[i] = bth[3 * i + 2];
+    }
+    return CB_OK;
+}
+
+int cb_extrapolate_gated(cb_plan* p, double t_target, void* const* outs, cb_dtype out_dtype, void* const* resid,
+                         cb_dtype resid_dtype, const void* const* gates, cb_dtype gate_dtype, void* stream) {
+    if (!p) return CB_ERR_ARG;
+    const int n = live_entries(p);
+    if (n == 0) return p->cache ? CB_ERR_HISTORY_NOT_FULL : CB_ERR_UNBOUND;
+    const Window win = live_window(p, n);
+    double w[CB_MAX_K];
+    const int rc = weights_for(p, win, t_target, w);
+    if (rc != CB_OK) return rc;
+    return run_launch(p, win, w, outs, out_dtype, resid, resid_dtype, stream, gates, gate_dtype);
+}
+
+int cb_cache_push_residual(cb_plan* p, const void* const* feats, cb_dtype feat_dtype, double t, void* const* resid,
+                           cb_dtype resid_dtype, const void* const* gates, cb_dtype gate_dtype, void* stream) {
+    if (!p || !feats || !valid_dtype(feat_dtype) || !valid_dtype(resid_dtype) || !std::isfinite(t))
+        return CB_ERR_ARG;
+    if (!p->cache) return CB_ERR_UNBOUND;
+    const int n = (int)p->tensors.size();
+    const int ng = (int)p->groups.size();
+    const size_t fes = esize(feat_dtype), res = esize(resid_dtype);
+    for (int i = 0; i < n; ++i) {
+        if (!feats[i]) return CB_ERR_ARG;
+        if (!aligned(feats[i], fes)) return CB_ERR_ALIGN;
+    }
+    if (resid)
+        for (int g = 0; g < ng; ++g)
+            if (resid[g] && !aligned(resid[g], res)) return CB_ERR_ALIGN;
+    int rc = check_gates(p, resid, gates, gate_dtype);
+    if (rc != CB_OK) return rc;
+    if (p->has_last) {
+        const double d = t - p->last_t;
+        if (d == 0.0 || (p->dir != 0 && (d > 0 ? 1 : -1) != p->dir)) return CB_ERR_ORDER;
+    }
+    for (int j = 0; j < p->count; ++j)
+        if (p->slot_t[(p->oldest() + j) % p->K] == t) return CB_ERR_NODES_DEGENERATE;
+
+    rc = ensure_device(p);
+    if (rc != CB_OK) return rc;
+    if (!p->status_clear) {
+        cudaError_t e = cudaMemsetAsync(p->status_word(), 0, sizeof(int), (cudaStream_t)stream);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
+        p->status_clear = true;
+    }
+    // one-entry history of weight 1: the new features themselves
+    Window one{};
+    one.n = 1;
+    const double w1[1] = {1.0};
+    rc = run_launch(p, one, w1, nullptr, p->cache_dtype, resid, resid_dtype, stream, gates, gate_dtype, feats,
+                    feat_dtype);
+    if (rc != CB_OK) return rc;
+    p->slot_t[p->next] = t;
+    p->next = (p->next + 1) % p->K;
+    if (p->count < p->K) ++p->count;
+    p->has_last = true;
+    p->last_t = t;
+    return CB_OK;
 }
 
 int cb_weights(const cb_plan* p, double t_target, double* w_logical) {

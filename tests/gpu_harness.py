@@ -126,7 +126,8 @@ class Walk:
 
     # ---- skipped step
     def extrapolate(self, t: float, out_dtype: str = "bf16", fused: bool = False, outs: bool = True,
-                    resid_dtype: str = "bf16", ring=None, salt: int = 0, explicit=None):
+                    resid_dtype: str = "bf16", ring=None, salt: int = 0, explicit=None, gates=None,
+                    gate_dtype: str = "bf16"):
         w = self.w
         out_t = [torch.empty(s.shape, dtype=TORCH[out_dtype], device=self.dev) for s in w.tensors] if outs else None
         resid = None
@@ -135,7 +136,10 @@ class Walk:
             resid = [workloads.hidden_state(w, g, self.dev, TORCH[resid_dtype], salt=salt)
                      for g in range(self.n_groups)]
             resid_host = [host(resid[g], self._gidx(g)) for g in range(self.n_groups)]
-        if explicit is not None:
+        if gates is not None:
+            cb.cb_extrapolate_gated(self.plan, t, out_t, CB[out_dtype], resid, CB[resid_dtype], gates,
+                                    CB[gate_dtype])
+        elif explicit is not None:
             cb.cb_extrapolate_weights(self.plan, explicit, out_t, CB[out_dtype], resid, CB[resid_dtype])
         elif ring is None:
             cb.cb_extrapolate(self.plan, t, out_t, CB[out_dtype], resid, CB[resid_dtype])
@@ -151,7 +155,7 @@ class Walk:
         return self.idx[i]
 
     def expected_and_compare(self, t, out_t, resid, resid_host, out_dtype="bf16", resid_dtype="bf16",
-                             times=None, nthreads=8, wts=None):
+                             times=None, nthreads=8, wts=None, G=None):
         """Oracle expectation for the live FIFO (or ``times`` relabelling it, or the
         explicit weights ``wts``) and the comparison."""
         w = self.w
@@ -173,11 +177,15 @@ class Walk:
             F = [[e[1][i] for e in entries] for i in members]
             X = resid_host[g] if g is not None else None
             x_dt = ORC[resid_dtype]
+            Gm = None if G is None else [G[i] for i in members]
             o64, r64 = orc.extrapolate(F, wts, cdt, orc.FP64, X=X, x_dtype=x_dt,
-                                       resid_dtype=orc.FP64 if g is not None else None, nthreads=nthreads)
+                                       resid_dtype=orc.FP64 if g is not None else None, nthreads=nthreads,
+                                       G=Gm)
             Fd = np.array([[bf16_to_f64(f) if cdt == orc.BF16 else f.astype(np.float64) for f in row]
                            for row in F])  # [nb, K, n]
             bound = np.einsum("j,bjn->bn", np.abs(wts), np.abs(Fd))
+            gbound = bound if Gm is None else np.array(
+                [bound[b] * (1.0 if Gm[b] is None else np.abs(Gm[b])) for b in range(len(members))])
             for b, i in enumerate(members):
                 if out_t is None:
                     continue
@@ -189,7 +197,7 @@ class Walk:
                     stats_out.append(compare_fp32(gpu, o64[b], float(np.max(np.abs(Fd[b])))))
             if g is not None:
                 gpu = host(resid[g], self.idx[members[0]])
-                rb = bound.sum(0) + np.abs(bf16_to_f64(X) if x_dt == orc.BF16 else X.astype(np.float64))
+                rb = gbound.sum(0) + np.abs(bf16_to_f64(X) if x_dt == orc.BF16 else X.astype(np.float64))
                 if resid_dtype == "bf16":
                     ref = orc.convert(r64, orc.FP64, orc.BF16)
                     stats_res.append(compare_bf16(gpu, ref, r64, rb))
@@ -221,3 +229,11 @@ def isfinite_all(*arrs):
 
 def log2(x):
     return math.log2(x) if x > 0 else float("-inf")
+
+
+def expand_gate(gate: torch.Tensor, shape, idx=None) -> np.ndarray:
+    """A [batch, hidden] gate broadcast over tokens to the tensor's elements (fp64)."""
+    b, t, h = shape
+    g = gate.detach().float().cpu().numpy().astype(np.float64)
+    full = np.broadcast_to(g[:, None, :], (b, t, h)).reshape(-1)
+    return full if idx is None else full[idx.cpu().numpy()]

@@ -204,3 +204,30 @@ def test_taylor_weights_match_oracle(cb, orc):
         cb.cb_taylor_weights([0.0, 1.0, 3.0], 4.0)  # not equispaced
     with pytest.raises(cb.CbError):
         cb.cb_taylor_weights([], 1.0)
+
+
+def test_shapes_and_gate_validation(cb):
+    st = cb.raw_status
+    arr = lambda *xs: (ctypes.c_void_p * len(xs))(*xs)
+    p = cb.cb_plan_create([999.0, 900.0], 2, [(0, 0, 2 * 4 * 8, 0), (0, 1, 2 * 4 * 8, 0), (1, 0, 64, -1)],
+                          cb.CB_BF16, 0.0, 999.0)
+    with pytest.raises(cb.CbError) as e:
+        cb.cb_plan_set_shapes(p, [(2, 4, 8), (2, 4, 8), (1, 1, 63)])  # product != numel
+    assert e.value.status == cb.CB_ERR_ARG
+    with pytest.raises(cb.CbError) as e:
+        cb.cb_plan_set_shapes(p, [(2, 4, 8), (4, 2, 8), (1, 1, 64)])  # one group, two shapes
+    assert e.value.status == cb.CB_ERR_ARG
+    cb.cb_plan_bind_cache(p, 0x100000, cb.cb_plan_cache_bytes(p))  # never dereferenced below
+    gates = arr(0x3000, 0, 0)
+    # history not full is reported before the gates are looked at
+    assert st("cb_extrapolate_gated", p, 800.0, None, 0, arr(0x5000), 0, gates, 0, None) == \
+        cb.CB_ERR_HISTORY_NOT_FULL
+    # pushes with gates validate shapes and alignment before launching
+    feats = arr(0x1000, 0x2000, 0x4000)
+    assert st("cb_cache_push_residual", p, feats, 0, 999.0, arr(0x5000), 0, gates, 0, None) == cb.CB_ERR_ARG
+    cb.cb_plan_set_shapes(p, [(2, 4, 8), (2, 4, 8), (1, 1, 64)])
+    assert st("cb_cache_push_residual", p, feats, 0, 999.0, arr(0x5000), 0, arr(0x3001, 0, 0), 0, None) == \
+        cb.CB_ERR_ALIGN
+    assert st("cb_cache_push_residual", p, feats, 0, 999.0, arr(0x5001), 0, gates, 0, None) == cb.CB_ERR_ALIGN
+    assert st("cb_cache_push_residual", p, feats, 0, 999.0, arr(0x5000), 0, gates, 9, None) == cb.CB_ERR_ARG
+    cb.cb_plan_destroy(p)

@@ -118,3 +118,104 @@ def test_shifted_flow_schedule(cb, H):
             stats.append(so)
     print("shifted schedule", H.merge(stats))
     walk.close()
+
+
+def _gates(w, dtype, seed, skip=()):
+    g = torch.Generator(device="cuda").manual_seed(seed)
+    out = []
+    for i, t in enumerate(w.tensors):
+        if i in skip:
+            out.append(None)
+            continue
+        b, _, h = t.shape
+        out.append((0.5 * torch.randn(b, h, generator=g, device="cuda")).to(dtype))
+    return out
+
+
+@pytest.mark.parametrize("kernel", ["bulk", "direct"])
+@pytest.mark.parametrize("resid_dtype", ["bf16", "fp32"])
+def test_gated_residual(cb, H, kernel, resid_dtype):
+    """x <- x + sum_b g_b * P_b with per-(batch, channel) gates broadcast over
+    tokens (a DiT block's adaLN gates applied to the un-gated cached outputs)."""
+    w = workloads.scaled(workloads.dit256(4), 8)
+    nodes = [w.timesteps[s] for s in (4, 8, 12, 16)]
+    walk = H.Walk(w, node_t=nodes, kernel=kernel)
+    cb.cb_plan_set_shapes(walk.plan, [t.shape for t in w.tensors])
+    for k, t in enumerate(nodes):
+        walk.push(t, k)
+    t = w.timesteps[18]
+    gates = _gates(w, torch.bfloat16, 11, skip={3, 10})
+    outs, resid, rh = walk.extrapolate(t, fused=True, gates=gates, resid_dtype=resid_dtype, salt=9)
+    G = [None if g is None else H.expand_gate(g, s.shape) for g, s in zip(gates, w.tensors)]
+    so, sr, _ = walk.expected_and_compare(t, outs, resid, rh, resid_dtype=resid_dtype, G=G)
+    _ok(so, "gated outs")
+    _ok(sr, ("gated resid", resid_dtype))
+    print("gated", kernel, resid_dtype, sr)
+    # gates of None everywhere: the gated entry equals cb_extrapolate bit for bit
+    a, ra, _ = walk.extrapolate(t, fused=True, salt=4)
+    b_, rb, _ = walk.extrapolate(t, fused=True, salt=4, gates=[None] * len(w.tensors))
+    for x, y in zip(ra, rb):
+        assert torch.equal(x.view(torch.int16), y.view(torch.int16))
+    walk.close()
+
+
+def test_gated_residual_odd_shapes(cb, H):
+    """Hidden sizes that are not multiples of 8 (scalar path), fp32 gates."""
+    from test_gpu_parity import _odd_workload
+    w = _odd_workload(4)
+    nodes = [950.0, 900.0, 850.0, 800.0]
+    walk = H.Walk(w, node_t=nodes)
+    cb.cb_plan_set_shapes(walk.plan, [t.shape for t in w.tensors])
+    for k, t in enumerate(nodes):
+        walk.push(t, k)
+    gates = _gates(w, torch.float32, 12)
+    outs, resid, rh = walk.extrapolate(760.0, fused=True, gates=gates, gate_dtype="fp32", salt=2)
+    G = [H.expand_gate(g, s.shape) for g, s in zip(gates, w.tensors)]
+    so, sr, _ = walk.expected_and_compare(760.0, outs, resid, rh, G=G)
+    _ok(so, "odd gated outs")
+    _ok(sr, "odd gated resid")
+    walk.close()
+
+
+@pytest.mark.parametrize("src", ["fp32", "bf16"])
+@pytest.mark.parametrize("odd", [False, True])
+def test_push_residual(cb, H, src, odd):
+    """Full step with the fused epilogue: the slots hold exactly what the plain
+    push writes, and x <- x + sum_b g_b f_b (un-rounded features) matches the
+    oracle's single rounding."""
+    from test_gpu_parity import _odd_workload
+    w = _odd_workload(3) if odd else workloads.scaled(workloads.pixart(), 32)
+    w.cache_dtype = "bf16"
+    nodes = [900.0, 800.0, 700.0]
+    a = H.Walk(w, K=3, node_t=nodes)
+    b = H.Walk(w, K=3, node_t=nodes)
+    cb.cb_plan_set_shapes(a.plan, [t.shape for t in w.tensors])
+    tdt = torch.float32 if src == "fp32" else torch.bfloat16
+    for k, t in enumerate(nodes):
+        feats = [workloads.trajectory(w, i, t, k, "cuda", out_dtype=tdt) for i in range(len(w.tensors))]
+        gates = _gates(w, torch.bfloat16, 20 + k, skip={0})
+        resid = [workloads.hidden_state(w, g, "cuda", salt=k) for g in range(a.n_groups)]
+        rh = [H.host(r) for r in resid]
+        cb.cb_cache_push_residual(a.plan, feats, H.CB[src], t, resid, cb.CB_BF16, gates, cb.CB_BF16)
+        cb.cb_cache_push(b.plan, feats, H.CB[src], t)
+        torch.cuda.synchronize()
+        # the slot just written holds identical bytes (padding and unwritten slots are not compared)
+        offs, slot = H.slot_layout([s_.numel for s_ in w.tensors], 2)
+        for i, s_ in enumerate(w.tensors):
+            lo = k * slot + offs[i]
+            assert torch.equal(a.cache[lo:lo + 2 * s_.numel], b.cache[lo:lo + 2 * s_.numel]), (k, i)
+        for g in range(a.n_groups):
+            members = [i for i, s in enumerate(w.tensors) if s.group == g]
+            F = [[H.host(feats[i])] for i in members]
+            G = [None if gates[i] is None else H.expand_gate(gates[i], w.tensors[i].shape) for i in members]
+            _, r64 = orc.extrapolate(F, [1.0], H.ORC[src], None, X=rh[g], x_dtype=orc.BF16,
+                                     resid_dtype=orc.FP64, G=G)
+            ref = orc.convert(r64, orc.FP64, orc.BF16)
+            Fd = np.array([f[0].astype(np.float64) if src == "fp32" else H.bf16_to_f64(f[0]) for f in F])
+            gb = np.array([np.ones_like(Fd[0]) if x is None else np.abs(x) for x in G])
+            bound = (gb * np.abs(Fd)).sum(0) + np.abs(H.bf16_to_f64(rh[g]))
+            st = H.compare_bf16(H.host(resid[g]), ref, r64, bound)
+            assert st["bad"] == 0, (g, st)
+            assert st["exact"] >= 0.99 * st["n"], st  # compensated sum: rounded once, like the oracle
+    a.close()
+    b.close()
