@@ -50,7 +50,8 @@ struct Shape {
     static constexpr int threads = consumers + 32;  // plus the producer warp
 };
 constexpr int kChunkBytes = 8192;   // one history entry's share of a tile
-constexpr int kBarrierBytes = 256;  // full[S] and empty[S] barriers, S <= 16
+constexpr int kBarrierBytes = 256;  // full[S] and empty[S] barriers, S <= kMaxStages
+static_assert(2 * 8 * kMaxStages <= kBarrierBytes, "barrier block holds every stage's barriers");
 constexpr unsigned long long kMinDrainNs = 10000000ull;  // copies land in microseconds
 constexpr unsigned long long kMaxWaitNs = 60000000000ull;  // no wait outlives a minute
 
@@ -146,7 +147,8 @@ __global__ void __launch_bounds__(Shape<CB16>::threads, 1)
     if (warp == NCW) {  // ---------------------------------- producer
         if (lane != 0) return;
         int it = 0;
-        unsigned u = 0;
+        unsigned u = 0;               // units issued
+        uint32_t ps = 0, wraps = 0;   // stage of the next unit; times the ring has wrapped
         bool ok = true;
         for (int tile = blockIdx.x; ok && tile < A.tiles_total; tile += gridDim.x) {
             while (tile >= A.tile_begin[it + 1]) ++it;
@@ -171,19 +173,24 @@ __global__ void __launch_bounds__(Shape<CB16>::threads, 1)
                 gsrc = (size_t)b0 * A.i_hidden[it] * gs;
                 gbytes = (uint32_t)((b1 - b0 + 1) * A.i_hidden[it] * gs);
             }
-            for (int m = 0; m < nb; ++m, ++u) {
-                const uint32_t stage = u % (unsigned)S, q = u / (unsigned)S;
-                if (q > 0 && !mbar_wait(empty0 + 8u * stage, (q - 1) & 1u, A.wait_ns)) {
+            for (int m = 0; m < nb; ++m) {
+                const uint32_t stage = ps;
+                if (wraps > 0 && !mbar_wait(empty0 + 8u * stage, (wraps - 1) & 1u, A.wait_ns)) {
                     record(A.status, 2);
                     ok = false;
                     break;
+                }
+                ++u;
+                if (++ps == (uint32_t)S) {
+                    ps = 0;
+                    ++wraps;
                 }
                 // the tile's bf16 hidden state travels with its last member
                 const bool with_x = GROUPED && A.stage_x && resid && full_tile && m == nb - 1;
                 const uint32_t xbytes = with_x ? (uint32_t)(TE * 2) : 0u;
                 const uint32_t gb = (GATED && A.m_gate[first + m]) ? gbytes : 0u;
                 mbar_expect_tx(full0 + 8u * stage, (uint32_t)K * bytes + xbytes + gb);
-                if (A.withhold_first && u == 0) continue;
+                if (A.withhold_first && u == 1) continue;
                 const uint32_t dst = buf0 + stage * stage_bytes;
                 if (bytes) {
 #pragma unroll
@@ -214,7 +221,7 @@ __global__ void __launch_bounds__(Shape<CB16>::threads, 1)
     auto chunk = [&](uint32_t stage, int j) { return stages + stage * stage_bytes + (size_t)j * kChunkBytes; };
     auto gate_stage = [&](uint32_t stage) -> const void* { return stages + stage * stage_bytes + (size_t)C * kChunkBytes; };
     int it = 0;
-    unsigned u = 0;
+    uint32_t cs = 0, cph = 0;  // stage of the next unit to consume and its phase parity
     for (int tile = blockIdx.x; tile < A.tiles_total; tile += gridDim.x) {
         while (tile >= A.tile_begin[it + 1]) ++it;
         const long long numel = A.numel[it];
@@ -229,7 +236,9 @@ __global__ void __launch_bounds__(Shape<CB16>::threads, 1)
         // state is written, so that its guarded elements can be recomputed
         const bool hold = GROUPED && full_tile && resid != nullptr;
         const bool mine = NV >= NCT || c < NV;  // fp32 tiles have fewer vectors than consumers
-        const unsigned u0 = u;
+        // stage of member m of this tile (nb < S: one wrap at most)
+        const uint32_t s0 = cs;
+        auto stage_of = [&](int m) { return s0 + m < (uint32_t)S ? s0 + m : s0 + m - (uint32_t)S; };
         long long ev[U];
 #pragma unroll
         for (int v = 0; v < U; ++v) ev[v] = e0 + ((long long)v * NCT + c) * kVecElems;
@@ -237,22 +246,20 @@ __global__ void __launch_bounds__(Shape<CB16>::threads, 1)
         // producer staged (or absolute, when gates stay in global memory)
         unsigned gi[U];
         if constexpr (GATED) {
-            if (hold && A.i_row[it] != 0) {  // items without a shape carry no gate
-                gate_offsets<U>(A, it, e0, ev, gi);
-                if (A.stage_gate_bytes) {
-                    const unsigned b0h = (unsigned)e0 / A.i_row[it] * A.i_hidden[it];  // gated: numel < 2^32
-#pragma unroll
-                    for (int v = 0; v < U; ++v) gi[v] -= b0h;
-                }
-            }
+            if (hold && A.i_row[it] != 0)  // items without a shape carry no gate
+                gate_offsets<U>(A, it, e0, ev, gi, A.stage_gate_bytes != 0);
         }
         Acc<U> acc;
         acc.zero();
-        for (int m = 0; m < nb; ++m, ++u) {
-            const uint32_t stage = u % (unsigned)S, q = u / (unsigned)S;
-            if (!mbar_wait(full0 + 8u * stage, q & 1u, A.wait_ns)) {
+        for (int m = 0; m < nb; ++m) {
+            const uint32_t stage = cs;
+            if (!mbar_wait(full0 + 8u * stage, cph, A.wait_ns)) {
                 record(A.status, 1);
                 return;
+            }
+            if (++cs == (uint32_t)S) {
+                cs = 0;
+                cph ^= 1u;
             }
             RawVecs<K, CB16, U> raw;
             if (full_tile && mine) {
@@ -314,7 +321,7 @@ __global__ void __launch_bounds__(Shape<CB16>::threads, 1)
             }
         }
         if (GROUPED && hold) {
-            const uint32_t last = (u0 + nb - 1) % (unsigned)S;
+            const uint32_t last = stage_of(nb - 1);
             auto xload = [&](int v, float (&x)[8]) {
                 if (A.stage_x)
                     unpack_bf16x8(*reinterpret_cast<const uint4*>(chunk(last, K) + (size_t)(ev[v] - e0) * 2), x);
@@ -330,7 +337,7 @@ __global__ void __launch_bounds__(Shape<CB16>::threads, 1)
                     const size_t off = (size_t)(ev[v] - e0 + e) * ES;
                     float tp = xe, tc = 0.0f;
                     for (int m = 0; m < nb; ++m) {
-                        const uint32_t st = (u0 + m) % (unsigned)S;
+                        const uint32_t st = stage_of(m);
                         float p = 0.0f, cc = 0.0f, h, l, qq;
 #pragma unroll
                         for (int j = 0; j < K; ++j) {
@@ -357,7 +364,7 @@ __global__ void __launch_bounds__(Shape<CB16>::threads, 1)
             }
             __syncwarp();
             if (lane == 0)
-                for (int m = 0; m < nb; ++m) mbar_arrive(empty0 + 8u * ((u0 + m) % (unsigned)S));
+                for (int m = 0; m < nb; ++m) mbar_arrive(empty0 + 8u * stage_of(m));
         } else if (!full_tile) {
             const long long end = e0 + TE < numel ? e0 + TE : numel;
             for (long long e = e0 + c; e < end; e += NCT) scalar_element<CB16>(A, K, it, e);

@@ -59,6 +59,8 @@ struct ExtrapArgs {
     const void* m_gate[kMaxMembers];    // gate [batch, hidden] of the member, or null (gate 1)
     unsigned i_hidden[kMaxItems];       // hidden size of the item's tensors
     unsigned i_row[kMaxItems];          // tokens * hidden of the item's tensors
+    unsigned long long i_hidden_magic[kMaxItems];  // ceil(2^64 / i_hidden) (0: i_hidden = 1)
+    unsigned long long i_row_magic[kMaxItems];     // ceil(2^64 / i_row) (0: i_row = 1)
 };
 
 // One full-step launch: copy/convert every tensor into one ring slot.
@@ -81,7 +83,9 @@ cudaError_t launch_extrapolate(const ExtrapArgs& a, int K, bool cache_bf16, int 
 cudaError_t launch_extrapolate_gated(const ExtrapArgs& a, int K, bool cache_bf16, int grid, cudaStream_t s);
 cudaError_t extrapolate_blocks_per_sm(int K, bool cache_bf16, int* blocks);
 
-// Bulk-copy pipeline variant (extrapolate_bulk.cu).
+// Bulk-copy pipeline variant (extrapolate_bulk.cu). Its barrier block holds
+// the full and empty barriers of at most kMaxStages stages.
+constexpr int kMaxStages = 16;
 size_t bulk_smem_bytes(int chunks_per_stage, size_t extra_per_stage, int stages);
 cudaError_t prepare_extrapolate_bulk(int K, bool cache_bf16, size_t smem);
 cudaError_t launch_extrapolate_bulk(const ExtrapArgs& a, int K, bool cache_bf16, int grid, size_t smem,

@@ -516,24 +516,37 @@ __device__ __forceinline__ void resid_precise(const ExtrapArgs& A, const long lo
     }
 }
 
+// n / d for n, d < 2^32 from M = ceil(2^64 / d) (M = 0 encodes d = 1):
+// n M / 2^64 = n / d + n delta / (d 2^64) with 0 <= delta < d, and the excess
+// n delta / (d 2^64) < 2^-32 < 1 / d cannot carry frac(n / d) <= (d - 1) / d
+// past the next integer (division by invariant integers, after Granlund &
+// Montgomery, PLDI 1994).
+__device__ __forceinline__ unsigned div_magic(unsigned n, unsigned long long M) {
+    return M ? (unsigned)__umul64hi((unsigned long long)n, M) : n;
+}
+
 // Gate offsets b * hidden + h of UV vectors of a tile starting at element e0
-// (32-bit arithmetic: gated tensors have fewer than 2^32 elements). Rows of
-// tokens * hidden are multiples of hidden, so h follows from e mod hidden.
+// (32-bit arithmetic: gated tensors have fewer than 2^32 elements); with
+// `relative`, b counts from the tile's first batch (the staged gate rows).
+// Rows of tokens * hidden are multiples of hidden, so h = e mod hidden.
 template <int UV>
 __device__ __forceinline__ void gate_offsets(const ExtrapArgs& A, int it, long long e0,
-                                             const long long (&ev)[UV], unsigned (&gi)[UV]) {
+                                             const long long (&ev)[UV], unsigned (&gi)[UV], bool relative = false) {
     const unsigned row = A.i_row[it], H = A.i_hidden[it], ue0 = (unsigned)e0;
-    const unsigned q0 = ue0 / row, r0 = ue0 - q0 * row, rh = r0 % H;
+    if (row == 0 || H == 0) {  // no shape: no gate
+#pragma unroll
+        for (int u = 0; u < UV; ++u) gi[u] = 0;
+        return;
+    }
+    const unsigned q0 = div_magic(ue0, A.i_row_magic[it]), r0 = ue0 - q0 * row;
 #pragma unroll
     for (int u = 0; u < UV; ++u) {
-        const unsigned off = (unsigned)(ev[u] - e0);
-        unsigned r = r0 + off, b = q0;
-        while (r >= row) {
+        unsigned r = r0 + (unsigned)(ev[u] - e0), b = relative ? 0u : q0;
+        while (r >= row) {  // a tile spans few rows
             r -= row;
             ++b;
         }
-        unsigned h = rh + off % H;
-        if (h >= H) h -= H;
+        const unsigned h = r - div_magic(r, A.i_hidden_magic[it]) * H;
         gi[u] = b * H + h;
     }
 }

@@ -143,9 +143,10 @@ int extrap_grid(cb_plan* p, int K, bool cb16, int tiles, int* grid) {
 // Largest gate staging per pipeline stage (two rows of 4096 fp32 channels).
 constexpr size_t kMaxStagedGateBytes = 32768;
 
-// Pipeline of the bulk kernel: as many stages of `chunks` 8 KB chunks as fit
-// in one CTA's shared memory (at most 8). The kernel's dynamic shared-memory
-// limit is raised to the device maximum once per instantiation.
+// Pipeline of the bulk kernel: as many stages of `chunks` 8 KB chunks (plus
+// `extra` bytes) as fit in one CTA's shared memory, at most kMaxStages. The
+// kernel's dynamic shared-memory limit is raised to the device maximum once
+// per instantiation.
 int bulk_config(cb_plan* p, int K, bool cb16, int chunks, size_t extra, bool gated, int* stages, size_t* smem) {
     int& prepared = gated ? p->dev.bulk_gated[cb16 ? 1 : 0][K] : p->dev.bulk_stages[cb16 ? 1 : 0][K];
     if (prepared == 0) {
@@ -154,7 +155,7 @@ int bulk_config(cb_plan* p, int K, bool cb16, int chunks, size_t extra, bool gat
         if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute");
         prepared = 1;
     }
-    int s = 8;
+    int s = cbk::kMaxStages;
     while (s > 1 && cbk::bulk_smem_bytes(chunks, extra, s) > (size_t)p->dev.smem_optin) --s;
     *stages = cbk::bulk_smem_bytes(chunks, extra, s) <= (size_t)p->dev.smem_optin ? s : 0;
     *smem = cbk::bulk_smem_bytes(chunks, extra, s);
@@ -176,6 +177,9 @@ int push_grid(cb_plan* p, bool sb, bool db, int tiles, int* grid) {
 }
 
 bool aligned(const void* ptr, size_t a) { return ((uintptr_t)ptr % a) == 0; }
+
+// Multiplier of the kernels' division by d < 2^32: ceil(2^64 / d), 0 for d <= 1.
+unsigned long long div_magic(unsigned d) { return d <= 1 ? 0ull : ~0ull / d + 1ull; }
 
 // Logical history window: n entries, oldest first, with the slot of each.
 struct Window {
@@ -310,6 +314,8 @@ int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs
         A.first[items] = (short)members;
         A.i_hidden[items] = (unsigned)p->sh_hidden[mem[0]];
         A.i_row[items] = (unsigned)(p->sh_tokens[mem[0]] * p->sh_hidden[mem[0]]);
+        A.i_hidden_magic[items] = div_magic(A.i_hidden[items]);
+        A.i_row_magic[items] = div_magic(A.i_row[items]);
         for (int m = 0; m < nm; ++m) {
             const int i = mem[m];
             void* o = feats ? slot + p->off[i] : outs ? outs[i] : nullptr;
