@@ -458,19 +458,27 @@ def run_e2e(args, torch, cb, wl, w, plan, cdt, tdt, dev, pushed, t_targets, byte
         outs = [torch.empty(t.shape, dtype=tdt, device=dev) for t in w.tensors]
         resid = [torch.empty_like(r, device=dev) for r in host_resid] if fused else None
 
+    split = []  # per step: (start, pushes done, end) events
+
     def step(k):
         cb.cb_plan_reset(plan)
         t = t_targets[k % len(t_targets)]
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+        split.append(ev)
         with torch.cuda.stream(stream):
+            ev[0].record(stream)
             if mode == "zerocopy":
                 for j, s in enumerate(nodes):
                     cb.cb_cache_push(plan, host_feats[j], cdt, w.timesteps[s], stream=stream)
+                ev[1].record(stream)
                 cb.cb_extrapolate(plan, t, host_outs, cdt, host_resid, cb.CB_BF16, stream=stream)
+                ev[2].record(stream)
                 return
             for j, s in enumerate(nodes):
                 for d, h in zip(dev_feats, host_feats[j]):
                     d.copy_(h, non_blocking=True)
                 cb.cb_cache_push(plan, dev_feats, cdt, w.timesteps[s], stream=stream)
+            ev[1].record(stream)
             if fused:
                 for d, h in zip(resid, host_resid):
                     d.copy_(h, non_blocking=True)
@@ -480,11 +488,13 @@ def run_e2e(args, torch, cb, wl, w, plan, cdt, tdt, dev, pushed, t_targets, byte
             if fused:
                 for h, d in zip(host_resid, resid):
                     h.copy_(d, non_blocking=True)
+            ev[2].record(stream)
 
     steps = max(1, args.e2e_steps)
     for k in range(2):
         step(k)
     stream.synchronize()
+    split.clear()
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     a.record(stream)
     for k in range(steps):
@@ -492,9 +502,12 @@ def run_e2e(args, torch, cb, wl, w, plan, cdt, tdt, dev, pushed, t_targets, byte
     b.record(stream)
     stream.synchronize()
     ms = max_over_ranks(a.elapsed_time(b) / steps, dev)
+    push_ms = sum(e[0].elapsed_time(e[1]) for e in split) / steps
+    extrap_ms = sum(e[1].elapsed_time(e[2]) for e in split) / steps
     return {"value": round(bytes_step * ws / (ms / 1e3) / 1e9, 2), "unit": "GB/s",
             "h2d_bytes_per_step": K * slot + resid_bytes, "d2h_bytes_per_step": slot + resid_bytes,
             "ms_per_step": round(ms, 3), "steps": steps, "mode": mode,
+            "push_ms": round(push_ms, 3), "extrapolate_ms": round(extrap_ms, 3),
             "path": "cb_cache_push x K from host buffers + cb_extrapolate into host buffers"}
 
 

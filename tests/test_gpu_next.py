@@ -177,6 +177,43 @@ def test_gated_residual_odd_shapes(cb, H):
     walk.close()
 
 
+# Gate-row cases of the bulk kernel's gate staging: batch rows that are not a
+# whole number of 4096-element tiles (a tile takes two gate rows), rows shorter
+# than a tile (gates stay in global memory), and hidden sizes whose two gate
+# rows fill (bf16) or overflow (fp32) the 32 KB staging limit.
+_GATE_CASES = {
+    "cross": [(4, 40, 1152)] * 3 + [(3, 24, 1024)] * 2,
+    "short": [(8, 2, 1152)] * 2 + [(5, 3, 512)] * 2,
+    "wide": [(2, 3, 8192)] * 2,
+}
+
+
+@pytest.mark.parametrize("case", sorted(_GATE_CASES))
+@pytest.mark.parametrize("gate_dtype", ["bf16", "fp32"])
+def test_gated_gate_rows(cb, H, case, gate_dtype):
+    shapes = _GATE_CASES[case]
+    groups = {}
+    tensors = []
+    for i, sh in enumerate(shapes):
+        g = groups.setdefault(sh, len(groups))
+        tensors.append(workloads.TensorSpec(g, i, sh, g))
+    w = workloads.Workload(name=f"gate-rows-{case}", tensors=tensors, K=4, cache_dtype="bf16", T=0, r=0,
+                           t_min=0.0, t_max=999.0, timesteps=[], degree=6, noise=0.1, seed=91)
+    nodes = [960.0, 900.0, 840.0, 780.0]
+    for kernel in ("bulk", "direct"):
+        walk = H.Walk(w, node_t=nodes, kernel=kernel)
+        cb.cb_plan_set_shapes(walk.plan, [t.shape for t in w.tensors])
+        for k, t in enumerate(nodes):
+            walk.push(t, k)
+        gates = _gates(w, H.TORCH[gate_dtype], 31, skip={1})
+        outs, resid, rh = walk.extrapolate(735.0, fused=True, gates=gates, gate_dtype=gate_dtype, salt=5)
+        G = [None if g is None else H.expand_gate(g, s.shape) for g, s in zip(gates, w.tensors)]
+        so, sr, _ = walk.expected_and_compare(735.0, outs, resid, rh, G=G)
+        _ok(so, (case, kernel, "outs"))
+        _ok(sr, (case, kernel, "resid"))
+        walk.close()
+
+
 @pytest.mark.parametrize("src", ["fp32", "bf16"])
 @pytest.mark.parametrize("odd", [False, True])
 def test_push_residual(cb, H, src, odd):
