@@ -1,15 +1,15 @@
 // Skipped-step kernel, bulk-copy pipeline variant (same arithmetic and bits as
-// extrapolate.cu; Sec. 3.3, Eq. for f_t; Alg. 1, extrapolation branch).
+// the direct kernel; Sec. 3.3, Eq. for f_t; Alg. 1, extrapolation branch).
 //
-// One CTA per SM. A producer lane moves, for every work unit (one tile of one
-// branch tensor), the K history chunks of 8 KB each from HBM into a ring of
-// shared-memory stages with cp.async.bulk (the Blackwell bulk-copy engine),
-// each stage guarded by a "full" mbarrier (transaction bytes) and an "empty"
-// mbarrier (one arrival per consumer warp). Consumer warps read their 8-element
-// vectors of the K chunks from shared memory, release the stage, and compute
-// and store from registers. With S stages of K x 8 KB (S = 5 for K = 5) up to
-// ~160 KB per SM stay in flight independently of the consumers' registers,
-// which is what bounds the direct-load variant.
+// One CTA per SM (two for K = 1). A producer lane moves,
+// for every work unit (one tile of one branch tensor), the K history chunks of
+// 8 KB each from HBM into a ring of shared-memory stages with cp.async.bulk
+// (the Blackwell bulk-copy engine), each stage guarded by a "full" mbarrier
+// (transaction bytes) and an "empty" mbarrier (one arrival per consumer warp).
+// Consumer warps read their 8-element vectors of the K chunks from shared
+// memory, compute, and store from registers. With S stages of K x 8 KB (S = 5
+// for K = 5) up to ~200 KB per SM stay in flight independently of the
+// consumers' registers, which is what bounds the direct-load variant.
 //
 // Every consumer thread takes one 8-element vector of a tile: 16 consumer
 // warps for bf16 tiles (17 warps, up to 96 registers per thread), 8 for fp32
@@ -42,10 +42,14 @@ namespace cbk {
 namespace {
 
 // One 8-element vector per consumer thread and tile: 16 consumer warps for
-// bf16 tiles (512 vectors), 8 for fp32 tiles (256 vectors).
-template <bool CB16>
+// bf16 tiles (512 vectors), 8 for fp32 tiles (256 vectors). One-entry
+// launches (K = 1: the full-step epilogue, or a single live entry) carry so
+// few bytes per unit that the consumers' fixed cost per unit dominates; they
+// run two CTAs of 8 consumer warps per SM (two independent pipelines), and
+// bf16 threads there take two vectors per tile.
+template <bool CB16, int K>
 struct Shape {
-    static constexpr int consumer_warps = CB16 ? 16 : 8;
+    static constexpr int consumer_warps = (CB16 && K > 1) ? 16 : 8;
     static constexpr int consumers = consumer_warps * 32;
     static constexpr int threads = consumers + 32;  // plus the producer warp
 };
@@ -116,11 +120,11 @@ __device__ __forceinline__ void record(int* status, int code) {
 // bookkeeping and with 16 consumer warps. GATED (with GROUPED): the hidden
 // state receives g_b * P_b, with a per-(batch, channel) gate per member.
 template <int K, bool CB16, bool GROUPED, bool GATED>
-__global__ void __launch_bounds__(Shape<CB16>::threads, 1)
+__global__ void __launch_bounds__(Shape<CB16, K>::threads, bulk_ctas_per_sm(K))
     extrapolate_bulk_kernel(const __grid_constant__ ExtrapArgs A) {
     extern __shared__ __align__(128) unsigned char smem[];
-    constexpr int NCW = Shape<CB16>::consumer_warps;
-    constexpr int NCT = Shape<CB16>::consumers;
+    constexpr int NCW = Shape<CB16, K>::consumer_warps;
+    constexpr int NCT = Shape<CB16, K>::consumers;
     constexpr long long TE = tile_elems(CB16);  // 8 KB per history chunk for both cache types
     constexpr int ES = CB16 ? 2 : 4;
     constexpr int NV = (int)(TE / kVecElems);     // vectors per tile: 512 (bf16) or 256 (fp32)

@@ -63,6 +63,7 @@ struct DeviceInfo {
     int device = -1;
     int sms = 0;
     int smem_optin = 0;                    // largest dynamic shared memory per CTA
+    int smem_per_sm = 0;                   // shared memory of one SM
     int occ_extrap[2][CB_MAX_K + 1] = {};  // [cache_bf16][K]
     int occ_push[2][2] = {};               // [src_bf16][dst_bf16]
     int bulk_stages[2][CB_MAX_K + 1] = {};  // 1 once the kernel's shared-memory limit is raised
@@ -121,6 +122,8 @@ int ensure_device(cb_plan* p) {
         if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
         e = cudaDeviceGetAttribute(&info.smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, d);
         if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
+        e = cudaDeviceGetAttribute(&info.smem_per_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, d);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
         p->dev = info;
     }
     return CB_OK;
@@ -155,9 +158,14 @@ int bulk_config(cb_plan* p, int K, bool cb16, int chunks, size_t extra, bool gat
         if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute");
         prepared = 1;
     }
+    // with several CTAs per SM each gets its share of the SM's shared memory
+    // (less the 1 KB the hardware reserves per CTA)
+    const int per_sm = cbk::bulk_ctas_per_sm(K);
+    size_t cap = (size_t)p->dev.smem_optin;
+    if (per_sm > 1) cap = std::min(cap, (size_t)p->dev.smem_per_sm / per_sm - 1024);
     int s = cbk::kMaxStages;
-    while (s > 1 && cbk::bulk_smem_bytes(chunks, extra, s) > (size_t)p->dev.smem_optin) --s;
-    *stages = cbk::bulk_smem_bytes(chunks, extra, s) <= (size_t)p->dev.smem_optin ? s : 0;
+    while (s > 1 && cbk::bulk_smem_bytes(chunks, extra, s) > cap) --s;
+    *stages = cbk::bulk_smem_bytes(chunks, extra, s) <= cap ? s : 0;
     *smem = cbk::bulk_smem_bytes(chunks, extra, s);
     return CB_OK;
 }
@@ -407,7 +415,8 @@ int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs
     rc = bulk_config(p, K, cb16, A.stage_chunks, A.stage_gate_bytes, any_gate, &A.stages, &smem);
     if (rc != CB_OK) return rc;
     if (A.stages < max_nb + 1) return launch_direct();  // too deep for shared memory
-    const int grid = (int)(tiles < p->dev.sms ? tiles : p->dev.sms);  // one CTA per SM
+    const long long ctas = (long long)p->dev.sms * cbk::bulk_ctas_per_sm(K);  // persistent grid
+    const int grid = (int)(tiles < ctas ? tiles : ctas);
     cudaError_t e = any_gate ? cbk::launch_extrapolate_bulk_gated(A, K, cb16, grid, smem, (cudaStream_t)stream)
                              : cbk::launch_extrapolate_bulk(A, K, cb16, grid, smem, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e, "extrapolate launch");
