@@ -148,7 +148,9 @@ def max_over_ranks(x: float, device) -> float:
 def workload_description(w) -> dict:
     slot = sum(t.numel for t in w.tensors) * w.esize()
     return {"workload": w.name, "tensors": len(w.tensors), "K": w.K, "storage": w.cache_dtype,
-            "slot_bytes": slot, "schedule": f"T={w.T}, full every r={w.r}"}
+            "slot_bytes": slot,
+            "schedule": (f"explicit nodes {list(w.explicit_nodes)}, targets {list(w.explicit_targets)}"
+                         if w.explicit_nodes else f"T={w.T}, full every r={w.r}")}
 
 
 def pick_window(w, orc):
@@ -278,8 +280,15 @@ def run_ours(args):
     if args.scale > 1:
         w = wl.scaled(w, args.scale)
     K = w.K
-    pushed, targets = pick_window(w, orc)
-    node_t = [w.timesteps[s] for s in orc.full_schedule(w.T, w.r, w.s0, w.s1, K).nonzero()[0]]
+    tiny = bool(w.explicit_nodes)
+    if tiny:  # explicit nodes and targets instead of a schedule; L2-resident, a latency case
+        w.timesteps = list(w.explicit_nodes) + list(w.explicit_targets)
+        pushed = list(range(len(w.explicit_nodes)))
+        targets = list(range(len(pushed), len(w.timesteps)))
+        node_t = list(w.explicit_nodes)
+    else:
+        pushed, targets = pick_window(w, orc)
+        node_t = [w.timesteps[s] for s in orc.full_schedule(w.T, w.r, w.s0, w.s1, K).nonzero()[0]]
     tensors = [(t.layer, t.branch, t.numel, t.group) for t in w.tensors]
     cdt = cb.CB_BF16 if w.cache_dtype == "bf16" else cb.CB_FP32
     tdt = torch.bfloat16 if w.cache_dtype == "bf16" else torch.float32
@@ -397,7 +406,7 @@ def run_ours(args):
 
     # ---- the whole online loop of Alg. 1 over the schedule, ring evolving
     sched = None
-    if args.step == "skip" and args.schedule_reps > 0:
+    if args.step == "skip" and args.schedule_reps > 0 and not tiny:
         sched = run_schedule_loop(args, torch, cb, wl, orc, w, plan, cdt, dev, stream, extrapolate_at, bytes_step)
 
     # ---- end to end through the public API with host buffers: upload the K
@@ -408,7 +417,7 @@ def run_ours(args):
         e2e = run_e2e(args, torch, cb, wl, w, plan, cdt, tdt, dev, pushed, t_targets, bytes_step, ws, fused)
 
     cpu = None
-    if rank == 0 and ws == 1 and not args.no_cpu and args.step == "skip":
+    if rank == 0 and ws == 1 and not args.no_cpu and args.step == "skip" and not tiny:
         host, wts, ti = sample_host_features(w, torch, wl, orc, args.cpu_elems, dev)
         threads = os.cpu_count() or 1
         gbs, n, reps, el = cpu_oracle_run(w, host, wts, args.cpu_seconds, threads)
@@ -425,7 +434,9 @@ def run_ours(args):
         desc.update({"bytes_per_step": bytes_step, "fused_residual": fused, "step": args.step,
                      "gated": bool(args.gated), "targets": targets,
                      "history_steps": pushed[-K:],
-                     "l2": "inputs larger than L2 (no flush)", "launch": "1 grouped persistent kernel per step",
+                     "l2": ("L2-resident inputs: a latency case (us_per_step), not a bandwidth one" if tiny
+                            else "inputs larger than L2 (no flush)"),
+                     "launch": "1 grouped persistent kernel per step",
                      "parallelism": f"replicas x{ws}" if ws > 1 else "1 GPU"})
         line = {
             "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": ws, "steps": args.steps,
@@ -592,7 +603,7 @@ def main():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
-    ap.add_argument("--config", default="flux", choices=["dit256", "dit256-k3", "dit512", "pixart", "flux"])
+    ap.add_argument("--config", default="flux", choices=["tiny", "dit256", "dit256-k3", "dit512", "pixart", "flux"])
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--fused", default="auto", choices=["auto", "on", "off"],
                     help="add the predictions into the blocks' hidden states (auto: as the workload states)")
