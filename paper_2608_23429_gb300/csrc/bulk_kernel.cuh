@@ -1,7 +1,7 @@
 // Skipped-step kernel, bulk-copy pipeline variant (same arithmetic and bits as
 // the direct kernel; Sec. 3.3, Eq. for f_t; Alg. 1, extrapolation branch).
 //
-// One CTA per SM (two for K = 1). A producer lane moves,
+// One or two CTAs per SM (see Shape). A producer lane moves,
 // for every work unit (one tile of one branch tensor), the K history chunks of
 // 8 KB each from HBM into a ring of shared-memory stages with cp.async.bulk
 // (the Blackwell bulk-copy engine), each stage guarded by a "full" mbarrier
@@ -42,14 +42,15 @@ namespace cbk {
 namespace {
 
 // One 8-element vector per consumer thread and tile: 16 consumer warps for
-// bf16 tiles (512 vectors), 8 for fp32 tiles (256 vectors). One-entry
-// launches (K = 1: the full-step epilogue, or a single live entry) carry so
-// few bytes per unit that the consumers' fixed cost per unit dominates; they
-// run two CTAs of 8 consumer warps per SM (two independent pipelines), and
-// bf16 threads there take two vectors per tile.
-template <bool CB16, int K>
+// bf16 tiles (512 vectors), 8 for fp32 tiles (256 vectors). Launches that
+// carry few bytes per unit (K = 1: the full-step epilogue or a single live
+// entry; bf16 predictions only with K <= 4) pay the consumers' fixed cost per
+// unit more often; they run two CTAs of 8 consumer warps per SM (two
+// independent pipelines), and bf16 threads there take two vectors per tile.
+template <bool CB16, int K, bool GROUPED>
 struct Shape {
-    static constexpr int consumer_warps = (CB16 && K > 1) ? 16 : 8;
+    static constexpr int ctas_per_sm = bulk_ctas_per_sm(K, CB16, GROUPED);
+    static constexpr int consumer_warps = (CB16 && ctas_per_sm == 1) ? 16 : 8;
     static constexpr int consumers = consumer_warps * 32;
     static constexpr int threads = consumers + 32;  // plus the producer warp
 };
@@ -120,11 +121,11 @@ __device__ __forceinline__ void record(int* status, int code) {
 // bookkeeping and with 16 consumer warps. GATED (with GROUPED): the hidden
 // state receives g_b * P_b, with a per-(batch, channel) gate per member.
 template <int K, bool CB16, bool GROUPED, bool GATED>
-__global__ void __launch_bounds__(Shape<CB16, K>::threads, bulk_ctas_per_sm(K))
+__global__ void __launch_bounds__(Shape<CB16, K, GROUPED>::threads, Shape<CB16, K, GROUPED>::ctas_per_sm)
     extrapolate_bulk_kernel(const __grid_constant__ ExtrapArgs A) {
     extern __shared__ __align__(128) unsigned char smem[];
-    constexpr int NCW = Shape<CB16, K>::consumer_warps;
-    constexpr int NCT = Shape<CB16, K>::consumers;
+    constexpr int NCW = Shape<CB16, K, GROUPED>::consumer_warps;
+    constexpr int NCT = Shape<CB16, K, GROUPED>::consumers;
     constexpr long long TE = tile_elems(CB16);  // 8 KB per history chunk for both cache types
     constexpr int ES = CB16 ? 2 : 4;
     constexpr int NV = (int)(TE / kVecElems);     // vectors per tile: 512 (bf16) or 256 (fp32)

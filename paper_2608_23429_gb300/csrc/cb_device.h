@@ -86,12 +86,17 @@ cudaError_t extrapolate_blocks_per_sm(int K, bool cache_bf16, int* blocks);
 // Bulk-copy pipeline variant (extrapolate_bulk.cu). Its barrier block holds
 // the full and empty barriers of at most kMaxStages stages.
 constexpr int kMaxStages = 16;
-// CTAs per SM of the bulk kernel: two for K = 1 (8 consumer warps each),
-// else one.
-__host__ __device__ constexpr int bulk_ctas_per_sm(int K) { return K == 1 ? 2 : 1; }
+// CTAs per SM of the bulk kernel (two of 8 consumer warps each, else one):
+// two for K = 1, and for bf16 prediction-only launches (not `grouped`) with
+// K <= 4, where two vectors per thread still fit the register budget.
+__host__ __device__ constexpr int bulk_ctas_per_sm(int K, bool src_bf16, bool grouped) {
+    return (K == 1 || (src_bf16 && !grouped && K <= 4)) ? 2 : 1;
+}
 size_t bulk_smem_bytes(int chunks_per_stage, size_t extra_per_stage, int stages);
 cudaError_t prepare_extrapolate_bulk(int K, bool cache_bf16, size_t smem);
-cudaError_t launch_extrapolate_bulk(const ExtrapArgs& a, int K, bool cache_bf16, int grid, size_t smem,
+// grouped: some item updates a hidden state or has several members (the
+// kernel's hidden-state bookkeeping); it also selects the CTA shape.
+cudaError_t launch_extrapolate_bulk(const ExtrapArgs& a, int K, bool cache_bf16, bool grouped, int grid, size_t smem,
                                     cudaStream_t s);
 // gated variant of the bulk kernel (extrapolate_bulk_gated.cu)
 cudaError_t prepare_extrapolate_bulk_gated(int K, bool cache_bf16, size_t smem);

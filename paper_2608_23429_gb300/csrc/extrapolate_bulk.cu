@@ -9,9 +9,9 @@ namespace {
 template <int K, bool CB16>
 cudaError_t launch_k(const ExtrapArgs& a, bool grouped, int grid, size_t smem, cudaStream_t s) {
     if (grouped)
-        extrapolate_bulk_kernel<K, CB16, true, false><<<grid, Shape<CB16, K>::threads, smem, s>>>(a);
+        extrapolate_bulk_kernel<K, CB16, true, false><<<grid, Shape<CB16, K, true>::threads, smem, s>>>(a);
     else
-        extrapolate_bulk_kernel<K, CB16, false, false><<<grid, Shape<CB16, K>::threads, smem, s>>>(a);
+        extrapolate_bulk_kernel<K, CB16, false, false><<<grid, Shape<CB16, K, false>::threads, smem, s>>>(a);
     return cudaGetLastError();
 }
 
@@ -54,10 +54,8 @@ cudaError_t prepare_extrapolate_bulk(int K, bool cache_bf16, size_t smem) {
 #undef P_F32
 }
 
-cudaError_t launch_extrapolate_bulk(const ExtrapArgs& a, int K, bool cache_bf16, int grid, size_t smem,
+cudaError_t launch_extrapolate_bulk(const ExtrapArgs& a, int K, bool cache_bf16, bool grouped, int grid, size_t smem,
                                     cudaStream_t s) {
-    bool grouped = false;
-    for (int i = 0; i < a.n_items; ++i) grouped = grouped || a.resid[i] != nullptr || a.nb[i] > 1;
 #define L_BF(k) launch_k<k, true>(a, grouped, grid, smem, s)
 #define L_F32(k) launch_k<k, false>(a, grouped, grid, smem, s)
     if (cache_bf16) {

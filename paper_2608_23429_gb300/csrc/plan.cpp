@@ -150,7 +150,8 @@ constexpr size_t kMaxStagedGateBytes = 32768;
 // `extra` bytes) as fit in one CTA's shared memory, at most kMaxStages. The
 // kernel's dynamic shared-memory limit is raised to the device maximum once
 // per instantiation.
-int bulk_config(cb_plan* p, int K, bool cb16, int chunks, size_t extra, bool gated, int* stages, size_t* smem) {
+int bulk_config(cb_plan* p, int K, bool cb16, bool grouped, int chunks, size_t extra, bool gated, int* stages,
+                size_t* smem) {
     int& prepared = gated ? p->dev.bulk_gated[cb16 ? 1 : 0][K] : p->dev.bulk_stages[cb16 ? 1 : 0][K];
     if (prepared == 0) {
         cudaError_t e = gated ? cbk::prepare_extrapolate_bulk_gated(K, cb16, (size_t)p->dev.smem_optin)
@@ -160,7 +161,7 @@ int bulk_config(cb_plan* p, int K, bool cb16, int chunks, size_t extra, bool gat
     }
     // with several CTAs per SM each gets its share of the SM's shared memory
     // (less the 1 KB the hardware reserves per CTA)
-    const int per_sm = cbk::bulk_ctas_per_sm(K);
+    const int per_sm = cbk::bulk_ctas_per_sm(K, cb16, grouped);
     size_t cap = (size_t)p->dev.smem_optin;
     if (per_sm > 1) cap = std::min(cap, (size_t)p->dev.smem_per_sm / per_sm - 1024);
     int s = cbk::kMaxStages;
@@ -351,15 +352,15 @@ int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs
         tiles += (numel + te - 1) / te;
         ++items;
     };
-    std::vector<char> grouped(n, 0);
+    std::vector<char> in_group(n, 0);
     if (resid)
         for (int g = 0; g < ng; ++g)
             if (resid[g] && !p->groups[g].empty()) {
                 add_item(p->groups[g].data(), (int)p->groups[g].size(), resid[g]);
-                for (int i : p->groups[g]) grouped[i] = 1;
+                for (int i : p->groups[g]) in_group[i] = 1;
             }
     for (int i = 0; i < n; ++i)
-        if (!grouped[i] && (feats || (outs && outs[i]))) add_item(&i, 1, nullptr);
+        if (!in_group[i] && (feats || (outs && outs[i]))) add_item(&i, 1, nullptr);
     if (tiles > 0x7FFFFFFFLL) return CB_ERR_LIMIT;
     A.tile_begin[items] = (int)tiles;
     A.n_items = items;
@@ -411,14 +412,17 @@ int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs
         }
         if (fits && need <= kMaxStagedGateBytes) A.stage_gate_bytes = (unsigned)((need + 127) / 128 * 128);
     }
+    // the grouped kernel (hidden-state bookkeeping) for gates, hidden states or multi-member items
+    bool grouped = any_gate;
+    for (int i = 0; i < items; ++i) grouped = grouped || A.resid[i] != nullptr || A.nb[i] > 1;
     size_t smem = 0;
-    rc = bulk_config(p, K, cb16, A.stage_chunks, A.stage_gate_bytes, any_gate, &A.stages, &smem);
+    rc = bulk_config(p, K, cb16, grouped, A.stage_chunks, A.stage_gate_bytes, any_gate, &A.stages, &smem);
     if (rc != CB_OK) return rc;
     if (A.stages < max_nb + 1) return launch_direct();  // too deep for shared memory
-    const long long ctas = (long long)p->dev.sms * cbk::bulk_ctas_per_sm(K);  // persistent grid
+    const long long ctas = (long long)p->dev.sms * cbk::bulk_ctas_per_sm(K, cb16, grouped);  // persistent grid
     const int grid = (int)(tiles < ctas ? tiles : ctas);
     cudaError_t e = any_gate ? cbk::launch_extrapolate_bulk_gated(A, K, cb16, grid, smem, (cudaStream_t)stream)
-                             : cbk::launch_extrapolate_bulk(A, K, cb16, grid, smem, (cudaStream_t)stream);
+                             : cbk::launch_extrapolate_bulk(A, K, cb16, grouped, grid, smem, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e, "extrapolate launch");
     return CB_OK;
 }
