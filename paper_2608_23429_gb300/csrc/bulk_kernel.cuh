@@ -47,9 +47,9 @@ namespace {
 // entry; bf16 predictions only with K <= 4) pay the consumers' fixed cost per
 // unit more often; they run two CTAs of 8 consumer warps per SM (two
 // independent pipelines), and bf16 threads there take two vectors per tile.
-template <bool CB16, int K, bool GROUPED>
+template <bool CB16, int K, bool GROUPED, bool GATED>
 struct Shape {
-    static constexpr int ctas_per_sm = bulk_ctas_per_sm(K, CB16, GROUPED);
+    static constexpr int ctas_per_sm = bulk_ctas_per_sm(K, CB16, GROUPED, GATED);
     static constexpr int consumer_warps = (CB16 && ctas_per_sm == 1) ? 16 : 8;
     static constexpr int consumers = consumer_warps * 32;
     static constexpr int threads = consumers + 32;  // plus the producer warp
@@ -121,11 +121,11 @@ __device__ __forceinline__ void record(int* status, int code) {
 // bookkeeping and with 16 consumer warps. GATED (with GROUPED): the hidden
 // state receives g_b * P_b, with a per-(batch, channel) gate per member.
 template <int K, bool CB16, bool GROUPED, bool GATED>
-__global__ void __launch_bounds__(Shape<CB16, K, GROUPED>::threads, Shape<CB16, K, GROUPED>::ctas_per_sm)
+__global__ void __launch_bounds__(Shape<CB16, K, GROUPED, GATED>::threads, Shape<CB16, K, GROUPED, GATED>::ctas_per_sm)
     extrapolate_bulk_kernel(const __grid_constant__ ExtrapArgs A) {
     extern __shared__ __align__(128) unsigned char smem[];
-    constexpr int NCW = Shape<CB16, K, GROUPED>::consumer_warps;
-    constexpr int NCT = Shape<CB16, K, GROUPED>::consumers;
+    constexpr int NCW = Shape<CB16, K, GROUPED, GATED>::consumer_warps;
+    constexpr int NCT = Shape<CB16, K, GROUPED, GATED>::consumers;
     constexpr long long TE = tile_elems(CB16);  // 8 KB per history chunk for both cache types
     constexpr int ES = CB16 ? 2 : 4;
     constexpr int NV = (int)(TE / kVecElems);     // vectors per tile: 512 (bf16) or 256 (fp32)

@@ -9,9 +9,9 @@ namespace {
 template <int K, bool CB16>
 cudaError_t launch_k(const ExtrapArgs& a, bool grouped, int grid, size_t smem, cudaStream_t s) {
     if (grouped)
-        extrapolate_bulk_kernel<K, CB16, true, false><<<grid, Shape<CB16, K, true>::threads, smem, s>>>(a);
+        extrapolate_bulk_kernel<K, CB16, true, false><<<grid, Shape<CB16, K, true, false>::threads, smem, s>>>(a);
     else
-        extrapolate_bulk_kernel<K, CB16, false, false><<<grid, Shape<CB16, K, false>::threads, smem, s>>>(a);
+        extrapolate_bulk_kernel<K, CB16, false, false><<<grid, Shape<CB16, K, false, false>::threads, smem, s>>>(a);
     return cudaGetLastError();
 }
 

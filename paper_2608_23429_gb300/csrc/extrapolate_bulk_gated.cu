@@ -7,7 +7,7 @@ namespace {
 
 template <int K, bool CB16>
 cudaError_t launch_gk(const ExtrapArgs& a, int grid, size_t smem, cudaStream_t s) {
-    extrapolate_bulk_kernel<K, CB16, true, true><<<grid, Shape<CB16, K, true>::threads, smem, s>>>(a);
+    extrapolate_bulk_kernel<K, CB16, true, true><<<grid, Shape<CB16, K, true, true>::threads, smem, s>>>(a);
     return cudaGetLastError();
 }
 

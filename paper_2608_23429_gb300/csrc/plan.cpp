@@ -147,11 +147,13 @@ int extrap_grid(cb_plan* p, int K, bool cb16, int tiles, int* grid) {
 constexpr size_t kMaxStagedGateBytes = 32768;
 
 // Pipeline of the bulk kernel: as many stages of `chunks` 8 KB chunks (plus
-// `extra` bytes) as fit in one CTA's shared memory, at most kMaxStages. The
-// kernel's dynamic shared-memory limit is raised to the device maximum once
-// per instantiation.
-int bulk_config(cb_plan* p, int K, bool cb16, bool grouped, int chunks, size_t extra, bool gated, int* stages,
-                size_t* smem) {
+// `extra` bytes) as fit in one CTA's shared memory, at most kMaxStages, and
+// the CTAs per SM. A shape made for two CTAs per SM runs one, with all of the
+// SM's shared memory, when half of it cannot hold `min_stages`. The kernel's
+// dynamic shared-memory limit is raised to the device maximum once per
+// instantiation.
+int bulk_config(cb_plan* p, int K, bool cb16, bool grouped, int chunks, size_t extra, bool gated, int min_stages,
+                int* stages, size_t* smem, int* ctas_per_sm) {
     int& prepared = gated ? p->dev.bulk_gated[cb16 ? 1 : 0][K] : p->dev.bulk_stages[cb16 ? 1 : 0][K];
     if (prepared == 0) {
         cudaError_t e = gated ? cbk::prepare_extrapolate_bulk_gated(K, cb16, (size_t)p->dev.smem_optin)
@@ -161,13 +163,16 @@ int bulk_config(cb_plan* p, int K, bool cb16, bool grouped, int chunks, size_t e
     }
     // with several CTAs per SM each gets its share of the SM's shared memory
     // (less the 1 KB the hardware reserves per CTA)
-    const int per_sm = cbk::bulk_ctas_per_sm(K, cb16, grouped);
-    size_t cap = (size_t)p->dev.smem_optin;
-    if (per_sm > 1) cap = std::min(cap, (size_t)p->dev.smem_per_sm / per_sm - 1024);
-    int s = cbk::kMaxStages;
-    while (s > 1 && cbk::bulk_smem_bytes(chunks, extra, s) > cap) --s;
-    *stages = cbk::bulk_smem_bytes(chunks, extra, s) <= cap ? s : 0;
-    *smem = cbk::bulk_smem_bytes(chunks, extra, s);
+    for (int per_sm = cbk::bulk_ctas_per_sm(K, cb16, grouped, gated); per_sm >= 1; --per_sm) {
+        size_t cap = (size_t)p->dev.smem_optin;
+        if (per_sm > 1) cap = std::min(cap, (size_t)p->dev.smem_per_sm / per_sm - 1024);
+        int s = cbk::kMaxStages;
+        while (s > 1 && cbk::bulk_smem_bytes(chunks, extra, s) > cap) --s;
+        *stages = cbk::bulk_smem_bytes(chunks, extra, s) <= cap ? s : 0;
+        *smem = cbk::bulk_smem_bytes(chunks, extra, s);
+        *ctas_per_sm = per_sm;
+        if (*stages >= min_stages) break;
+    }
     return CB_OK;
 }
 
@@ -416,10 +421,12 @@ int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs
     bool grouped = any_gate;
     for (int i = 0; i < items; ++i) grouped = grouped || A.resid[i] != nullptr || A.nb[i] > 1;
     size_t smem = 0;
-    rc = bulk_config(p, K, cb16, grouped, A.stage_chunks, A.stage_gate_bytes, any_gate, &A.stages, &smem);
+    int per_sm = 1;
+    rc = bulk_config(p, K, cb16, grouped, A.stage_chunks, A.stage_gate_bytes, any_gate, max_nb + 1, &A.stages,
+                     &smem, &per_sm);
     if (rc != CB_OK) return rc;
     if (A.stages < max_nb + 1) return launch_direct();  // too deep for shared memory
-    const long long ctas = (long long)p->dev.sms * cbk::bulk_ctas_per_sm(K, cb16, grouped);  // persistent grid
+    const long long ctas = (long long)p->dev.sms * per_sm;  // persistent grid
     const int grid = (int)(tiles < ctas ? tiles : ctas);
     cudaError_t e = any_gate ? cbk::launch_extrapolate_bulk_gated(A, K, cb16, grid, smem, (cudaStream_t)stream)
                              : cbk::launch_extrapolate_bulk(A, K, cb16, grouped, grid, smem, (cudaStream_t)stream);
