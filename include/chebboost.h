@@ -116,7 +116,7 @@ enum {
  * Errors: CB_ERR_ARG for T <= 0, r <= 0, s0 < 0, s1 < 0, K < 0 or is_full NULL. */
 int cb_schedule_full(int T, int r, int s0, int s1, int K, uint8_t* is_full, int* n_full);
 
-/* Offline precomputation (Sec. 3.3 "Weight Precomputation"; Alg. 1, offline
+/* Offline precomputation (the weight precomputation of Sec. 3.3; Alg. 1, offline
  * stage). node_t: host array of the n_nodes timesteps at which full
  * computations happen, in sampling order (strictly monotone). For every
  * window of K consecutive nodes the fp64 barycentric weights rho_j of

@@ -10,8 +10,8 @@
  *
  * Functions and the passages they follow:
  *   orc_full_schedule   Sec. 3.3, Eq. for the full-computation set F, plus the
- *                       warm-up reading of Sec. 3.3 "provided the history
- *                       buffer H contains enough entries (|H| = n)".
+ *                       warm-up reading of Sec. 3.3: a step extrapolates only
+ *                       once the history buffer H holds n entries.
  *   orc_normalize       Sec. 3.3: timesteps mapped affinely onto [-1, 1].
  *   orc_nodal           App. A: nodal polynomial omega(x) = prod_k (x - x_k).
  *   orc_rho             App. A, Eq. general_weights: rho_j = 1 / omega'(x_j),
@@ -29,8 +29,8 @@
  *                       residual of Sec. 3.1 (B(x) = x + S + C + M): the hidden
  *                       state plus every branch prediction, each optionally
  *                       times its per-element gate, rounded once.
- *   orc_convert         the cache write of Alg. 1 ("store the pair in H"):
- *                       a copy, or fp32 -> bf16 round-to-nearest-even.
+ *   orc_convert         the cache write of Alg. 1 (the full step's pair goes
+ *                       into H): a copy, or fp32 -> bf16 round-to-nearest-even.
  *   orc_bf16_encode /   bf16 <-> fp64 from the IEEE-754 bit layout (8 exponent
  *   orc_bf16_decode     bits, 7 stored fraction bits), round-to-nearest-even.
  *

@@ -11,11 +11,8 @@
 // for K = 5) up to ~200 KB per SM stay in flight independently of the
 // consumers' registers, which is what bounds the direct-load variant.
 //
-// Every consumer thread takes one 8-element vector of a tile: 16 consumer
-// warps for bf16 tiles (17 warps, up to 96 registers per thread), 8 for fp32
-// tiles. Many warps per scheduler hide the consumers' fixed latencies; the
-// arithmetic per byte is high enough that 8 warps with two vectors each
-// leave the grouped launches issue-bound. Two kinds of launch (GROUPED):
+// Many consumer warps per scheduler hide the consumers' fixed latencies (see
+// Shape for the thread map). Two kinds of launch (GROUPED):
 //   * predictions only: each stage is released as soon as it is in
 //     registers, and guarded elements are recomputed from registers;
 //   * with hidden states: stages are released after the member's arithmetic,
@@ -27,6 +24,9 @@
 //     producer). With gates, each member's stage also carries the gate rows
 //     of the batches its tile touches, so that no consumer waits on a global
 //     load.
+// The same kernel runs a full step's epilogue (cb_cache_push_residual) as a
+// one-entry history of weight 1 whose member addresses are the new features;
+// with copy_out the outputs (the ring slot) receive the features converted.
 //
 // Every wait is bounded (%globaltimer). A wait that runs out records a code in
 // the plan's device status word and the thread returns; the producer then
@@ -41,12 +41,14 @@
 namespace cbk {
 namespace {
 
-// One 8-element vector per consumer thread and tile: 16 consumer warps for
-// bf16 tiles (512 vectors), 8 for fp32 tiles (256 vectors). Launches that
-// carry few bytes per unit (K = 1: the full-step epilogue or a single live
-// entry; bf16 predictions only with K <= 4) pay the consumers' fixed cost per
-// unit more often; they run two CTAs of 8 consumer warps per SM (two
-// independent pipelines), and bf16 threads there take two vectors per tile.
+// Thread map. With one CTA per SM, one 8-element vector per consumer thread
+// and tile: 16 consumer warps for bf16 tiles (512 vectors; 17 warps cap
+// registers at 96), 8 for fp32 tiles (256 vectors). Launches that carry few
+// bytes per unit (K = 1, and bf16 launches with small K: bulk_ctas_per_sm) pay
+// the consumers' fixed cost per unit more often; they run two CTAs of 8
+// consumer warps per SM (two independent pipelines), bf16 threads taking two
+// vectors per tile. An earlier map of 8 consumer warps with two vectors each
+// on one CTA left the launches with hidden states issue-bound.
 template <bool CB16, int K, bool GROUPED, bool GATED>
 struct Shape {
     static constexpr int ctas_per_sm = bulk_ctas_per_sm(K, CB16, GROUPED, GATED);
@@ -116,10 +118,10 @@ __device__ __forceinline__ void record(int* status, int code) {
     if (status) atomicOr(status, code);
 }
 
-// GROUPED: some item updates a hidden state (stage holding, hidden-state
-// staging, 8 consumer warps); prediction-only launches compile without that
-// bookkeeping and with 16 consumer warps. GATED (with GROUPED): the hidden
-// state receives g_b * P_b, with a per-(batch, channel) gate per member.
+// GROUPED: some item updates a hidden state or has several members (stage
+// holding, hidden-state staging); prediction-only launches compile without
+// that bookkeeping. GATED (with GROUPED): the hidden state receives g_b * P_b,
+// with a per-(batch, channel) gate per member.
 template <int K, bool CB16, bool GROUPED, bool GATED>
 __global__ void __launch_bounds__(Shape<CB16, K, GROUPED, GATED>::threads, Shape<CB16, K, GROUPED, GATED>::ctas_per_sm)
     extrapolate_bulk_kernel(const __grid_constant__ ExtrapArgs A) {
@@ -210,13 +212,17 @@ __global__ void __launch_bounds__(Shape<CB16, K, GROUPED, GATED>::threads, Shape
                              full0 + 8u * stage);
             }
         }
-        // never leave while copies into this CTA's shared memory are in flight
-        const unsigned long long drain_ns = A.wait_ns > kMinDrainNs ? A.wait_ns : kMinDrainNs;
+        // never leave while copies into this CTA's shared memory are in flight:
+        // wait for every unit still in the ring; after one wait runs out (a unit
+        // whose copies were never issued) the others get the short limit
+        unsigned long long drain_ns = A.wait_ns > kMinDrainNs ? A.wait_ns : kMinDrainNs;
+        bool drained = true;
         for (unsigned q = u > (unsigned)S ? u - S : 0; q < u; ++q)
             if (!mbar_wait(full0 + 8u * (q % S), (q / S) & 1u, drain_ns)) {
-                record(A.status, 4);
-                break;
+                drained = false;
+                drain_ns = kMinDrainNs;
             }
+        if (!drained) record(A.status, 4);
         return;
     }
 

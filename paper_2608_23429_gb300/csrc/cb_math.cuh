@@ -1,6 +1,6 @@
 // Internal: the per-element arithmetic of the skipped-step kernels, shared by
-// the direct-load kernel (extrapolate.cu) and the bulk-copy pipeline kernel
-// (extrapolate_bulk.cu) so that both produce identical bits.
+// the direct-load kernel (direct_kernel.cuh) and the bulk-copy pipeline kernel
+// (bulk_kernel.cuh) so that both produce identical bits.
 //
 // Fast path. s = sum_j w_hi[j] F_j by fp32 FMA and, alongside,
 // a = sum_j |w_hi[j]| |F_j|. With u = 2^-24 the FMA chain plus the dropped low

@@ -1,9 +1,9 @@
-// Host side of libchebboost: the plan (offline precomputation, Sec. 3.3
-// "Weight Precomputation"; Alg. 1 offline stage), the history buffer's ring
-// bookkeeping, the online weights (Sec. 3.2 Eq. barycentric_coeff) and the
-// launches of the two kernels. Everything here is fp64 host arithmetic that
-// runs in microseconds per call; all device work is in push.cu and
-// extrapolate.cu.
+// Host side of libchebboost: the plan (the offline weight precomputation of
+// Sec. 3.3; Alg. 1 offline stage), the history buffer's ring bookkeeping, the
+// online weights (Sec. 3.2 Eq. barycentric_coeff) and the kernel launches.
+// Everything here is fp64 host arithmetic that runs in microseconds per call;
+// all device work is in push.cu and the extrapolate*.cu instantiations of the
+// skipped-step kernels.
 #include <cuda_runtime.h>
 
 #include <algorithm>
