@@ -591,10 +591,25 @@ def run_e2e(args, torch, cb, wl, w, plan, cdt, tdt, dev, pushed, t_targets, byte
     ms = max_over_ranks(a.elapsed_time(b) / steps, dev)
     push_ms = sum(e[0].elapsed_time(e[1]) for e in split) / steps
     extrap_ms = sum(e[1].elapsed_time(e[2]) for e in split) / steps
+    # the host link's own bound: one large pinned host -> device copy
+    link = torch.empty(1 << 30, dtype=torch.uint8).pin_memory()
+    link_dev = torch.empty(link.numel(), dtype=torch.uint8, device=dev)
+    with torch.cuda.stream(stream):
+        link_dev.copy_(link, non_blocking=True)
+        a.record(stream)
+        for _ in range(3):
+            link_dev.copy_(link, non_blocking=True)
+        b.record(stream)
+    stream.synchronize()
+    link_gbs = 3 * link.numel() / (a.elapsed_time(b) / 1e3) / 1e9
+    del link, link_dev
+    h2d, d2h = K * slot + resid_bytes, slot + resid_bytes
     return {"value": round(bytes_step * ws / (ms / 1e3) / 1e9, 2), "unit": "GB/s",
-            "h2d_bytes_per_step": K * slot + resid_bytes, "d2h_bytes_per_step": slot + resid_bytes,
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
             "ms_per_step": round(ms, 3), "steps": steps, "mode": mode,
             "push_ms": round(push_ms, 3), "extrapolate_ms": round(extrap_ms, 3),
+            "host_link_gbs": round(link_gbs, 1),
+            "frac_of_host_link": round((h2d + d2h) / (ms / 1e3) / 1e9 / link_gbs, 4),
             "path": "cb_cache_push x K from host buffers + cb_extrapolate into host buffers"}
 
 
