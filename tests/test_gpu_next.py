@@ -214,6 +214,34 @@ def test_gated_gate_rows(cb, H, case, gate_dtype):
         walk.close()
 
 
+@pytest.mark.parametrize("K", [1, 2, 3, 6, 8])
+def test_gated_every_history_size(cb, H, K):
+    """The gated kernels at every history size class (one and two CTAs per SM,
+    with and without spilled registers), both kernels, staged gate rows."""
+    shapes = _GATE_CASES["cross"]
+    groups = {}
+    tensors = []
+    for i, sh in enumerate(shapes):
+        g = groups.setdefault(sh, len(groups))
+        tensors.append(workloads.TensorSpec(g, i, sh, g))
+    w = workloads.Workload(name=f"gated-k{K}", tensors=tensors, K=K, cache_dtype="bf16", T=0, r=0,
+                           t_min=0.0, t_max=999.0, timesteps=[], degree=6, noise=0.1, seed=92 + K)
+    nodes = [980.0 - 41.0 * k for k in range(K)]
+    for kernel in ("bulk", "direct"):
+        walk = H.Walk(w, node_t=nodes, kernel=kernel)
+        cb.cb_plan_set_shapes(walk.plan, [t.shape for t in w.tensors])
+        for k, t in enumerate(nodes):
+            walk.push(t, k)
+        gates = _gates(w, torch.bfloat16, 40 + K, skip={2})
+        t = nodes[-1] - 25.0
+        outs, resid, rh = walk.extrapolate(t, fused=True, gates=gates, salt=K)
+        G = [None if g is None else H.expand_gate(g, s.shape) for g, s in zip(gates, w.tensors)]
+        so, sr, _ = walk.expected_and_compare(t, outs, resid, rh, G=G)
+        _ok(so, (K, kernel, "outs"))
+        _ok(sr, (K, kernel, "resid"))
+        walk.close()
+
+
 @pytest.mark.parametrize("src", ["fp32", "bf16"])
 @pytest.mark.parametrize("odd", [False, True])
 def test_push_residual(cb, H, src, odd):

@@ -246,7 +246,8 @@ def test_ring_variant_and_rotation_bit_exact(cb, H):
 
 # ------------------------------------------------------------- edge cases
 @pytest.mark.parametrize("kernel", ["direct", "bulk"])
-@pytest.mark.parametrize("K,cache", [(1, "bf16"), (2, "fp32"), (5, "bf16"), (8, "bf16"), (8, "fp32")])
+@pytest.mark.parametrize("K,cache", [(1, "bf16"), (1, "fp32"), (2, "bf16"), (2, "fp32"), (3, "bf16"), (5, "bf16"),
+                                     (6, "bf16"), (7, "fp32"), (8, "bf16"), (8, "fp32")])
 def test_odd_sizes_every_element(cb, H, K, cache, kernel):
     w = _odd_workload(K, cache)
     nodes = [990.0 - 37.0 * k for k in range(K)]
