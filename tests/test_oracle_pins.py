@@ -342,6 +342,34 @@ def test_gated_residual(orc):
     assert np.array_equal(r1, r0)
 
 
+def test_gated_pin_catches_planted_mistakes(orc):
+    """The gated-residual pin (numpy x + sum_b g_b P_b) rejects the plausible
+    mistakes, each planted in the oracle's inputs on the CPU: gates swapped
+    between members, the gate also scaling the hidden state, a member's gate
+    dropped, the hidden state dropped."""
+    rng = np.random.default_rng(25)
+    K, n = 3, 2000
+    F = [[rng.standard_normal(n).astype(np.float32) for _ in range(K)] for _ in range(2)]
+    X = rng.standard_normal(n).astype(np.float32)
+    w = rng.standard_normal(K)
+    G = [rng.standard_normal(n), rng.standard_normal(n)]
+    P = np.einsum("j,bjn->bn", w, np.array(F, np.float64))
+    ref = X.astype(np.float64) + G[0] * P[0] + G[1] * P[1]
+
+    def res(F_, X_, G_):
+        return orc.extrapolate(F_, w, orc.FP32, None, X=X_, x_dtype=orc.FP32, resid_dtype=orc.FP64, G=G_)[1]
+
+    assert _rel(res(F, X, G), ref) <= 1e-14
+    planted = {
+        "swapped gates": res(F, X, G[::-1]),
+        "gate on x": res(F, (X * G[0]).astype(np.float32), G),
+        "dropped gate": res(F, X, [G[0], None]),
+        "dropped x": res(F, np.zeros_like(X), G),
+    }
+    for name, r in planted.items():
+        assert _rel(r, ref) > 1e-6, name
+
+
 def test_threads_identical(orc):
     rng = np.random.default_rng(19)
     F = [orc.bf16_encode(rng.standard_normal(10001)) for _ in range(5)]
