@@ -32,7 +32,7 @@ struct ExtrapArgs {
     long long slot_off[8];       // byte offset of history entry j (0 = oldest)
     float w_hi[8];               // fp32(w_j)
     float w_lo[8];               // fp32(w_j - w_hi[j])
-    float w_abs[8];              // |w_hi[j]| (error bound of the fast path)
+    float w_guard[8];            // (K+2) u (1.01) 2^9 |w_hi[j]|: the fast path's scaled error bound
     int n_items;
     int tiles_total;
     int out_bf16;    // predictions are bf16 (else fp32)

@@ -6,7 +6,10 @@
 // a = sum_j |w_hi[j]| |F_j|. With u = 2^-24 the FMA chain plus the dropped low
 // half of each weight give |s - P| <= (K+1) u a (1 + O(Ku)). Whenever
 // (K+2) u a (1.01) <= 2^-9 |s| that error is below the smallest bf16 spacing
-// next to s, so bf16(s) lies within one bf16 ulp of bf16(P) (guard_ok).
+// next to s, so bf16(s) lies within one bf16 ulp of bf16(P). The kernels
+// accumulate the bound already scaled, a' = sum_j w_guard[j] |F_j| with
+// w_guard[j] = (K+2) u (1.01) 2^9 |w_hi[j]| (host-computed), so the test is
+// a' <= |s|; the 1 % margin covers the extra fp32 roundings of a'.
 // Elements failing the test (strong cancellation, ~1e-4..3e-3 of them) are
 // recomputed from the values already loaded with Dot2 (Ogita, Rump &
 // Oishi, "Accurate Sum and Dot Product", SIAM J. Sci. Comput. 26(6), 2005:
@@ -337,8 +340,15 @@ __device__ __forceinline__ void exact_from_raw(const ExtrapArgs& A, const RawVec
 // (K+2) u a (1.01) <= 2^-9 |s| keeps the interval between s and P shorter than
 // the smallest bf16 spacing next to s (2^-8 |s| in s's binade, 2^-9 |s| below
 // it), so it holds at most one rounding midpoint and bf16(s) is within one ulp
-// of bf16(P).
-__device__ __forceinline__ bool guard_ok(float g, float a, float s) { return g * a <= 0x1.0p-9f * fabsf(s); }
+// of bf16(P). With the scaled bound a' (see above) the test is a' <= |s|.
+__device__ __forceinline__ bool guard_ok(float a_scaled, float s) { return a_scaled <= fabsf(s); }
+
+// s0, s1 += w * (f0, f1): one paired fp32 FMA, each lane rounded like fmaf.
+__device__ __forceinline__ void fma_pair(float w, float f0, float f1, float& s0, float& s1) {
+    const float2 r = __ffma2_rn(make_float2(w, w), make_float2(f0, f1), make_float2(s0, s1));
+    s0 = r.x;
+    s1 = r.y;
+}
 
 // Fast path for one member over UV aligned 8-element vectors already loaded
 // into registers: bf16 prediction (if out) and accumulation into acc. The
@@ -353,7 +363,6 @@ template <int K, bool CB16, int UV, bool FROM_RAW, bool GATED = false, typename 
 __device__ __forceinline__ void member_fast(const ExtrapArgs& A, long long moff, void* out,
                                             const long long (&ev)[UV], const RawVecs<K, CB16, UV>& raw,
                                             bool accumulate, Acc<UV>& acc, Gate gate = {}, Exact exact = {}) {
-    const float g_out = (float)(K + 2) * kU * 1.01f;
 #pragma unroll
     for (int u = 0; u < UV; ++u) {
         float s[8], a[8];
@@ -364,10 +373,9 @@ __device__ __forceinline__ void member_fast(const ExtrapArgs& A, long long moff,
             float f[8];
             unpack<CB16>(raw[u][j], f);
 #pragma unroll
-            for (int e = 0; e < 8; ++e) {
-                s[e] = fmaf(A.w_hi[j], f[e], s[e]);
-                a[e] = fmaf(A.w_abs[j], fabsf(f[e]), a[e]);
-            }
+            for (int e = 0; e < 8; e += 2) fma_pair(A.w_hi[j], f[e], f[e + 1], s[e], s[e + 1]);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) a[e] = fmaf(A.w_guard[j], fabsf(f[e]), a[e]);
         }
         if (out) {
             uint32_t pk[4];
@@ -375,7 +383,7 @@ __device__ __forceinline__ void member_fast(const ExtrapArgs& A, long long moff,
             for (int i = 0; i < 4; ++i) pk[i] = pack_bf16x2(s[2 * i], s[2 * i + 1]);
             unsigned bad = 0;
 #pragma unroll
-            for (int e = 0; e < 8; ++e) bad |= guard_ok(g_out, a[e], s[e]) ? 0u : (1u << e);
+            for (int e = 0; e < 8; ++e) bad |= guard_ok(a[e], s[e]) ? 0u : (1u << e);
             while (bad) {  // rare: recompute the failing elements with Dot2
                 const int e = __ffs(bad) - 1;
                 bad &= bad - 1;
@@ -395,7 +403,7 @@ __device__ __forceinline__ void member_fast(const ExtrapArgs& A, long long moff,
             if constexpr (GATED) gate(u, g);
 #pragma unroll
             for (int e = 0; e < 8; ++e) {
-                if constexpr (GATED) {  // x + g * s: one rounding, bound |g| a
+                if constexpr (GATED) {  // x + g * s: one rounding, bound |g| a'
                     acc.x[u][e] = fmaf(g[e], s[e], acc.x[u][e]);
                     acc.y[u][e] = fmaf(fabsf(g[e]), a[e], acc.y[u][e]);
                 } else {
@@ -413,7 +421,12 @@ __device__ __forceinline__ void member_fast(const ExtrapArgs& A, long long moff,
 template <int K, int UV, typename XLoad, typename Exact>
 __device__ __forceinline__ void resid_fast(const ExtrapArgs& A, int it, const long long (&ev)[UV],
                                            const Acc<UV>& acc, void* resid, XLoad xload, Exact exact) {
-    const float g_res = (float)(K + A.nb[it] + 3) * kU * 1.01f;
+    // the test g_res (sum_b a_b + |x|) <= 2^-9 |t|, g_res = (K + nb + 3) u 1.01,
+    // on the scaled bounds acc.y = (K+2) u 1.01 2^9 sum_b a_b:
+    // q acc.y + r |x| <= |t| with q = (K + nb + 3) / (K + 2), r = g_res 2^9
+    const float kn = (float)(K + A.nb[it] + 3);
+    const float q = kn * (1.0f / (float)(K + 2)) * 1.0000005f;  // rounded up past fp32 error
+    const float r = kn * (kU * 1.01f * 512.0f);
 #pragma unroll
     for (int u = 0; u < UV; ++u) {
         float x[8], t[8];
@@ -423,9 +436,17 @@ __device__ __forceinline__ void resid_fast(const ExtrapArgs& A, int it, const lo
         for (int e = 0; e < 8; ++e) t[e] = acc.x[u][e] + x[e];
 #pragma unroll
         for (int i = 0; i < 4; ++i) pk[i] = pack_bf16x2(t[2 * i], t[2 * i + 1]);
-        unsigned bad = 0;
+        float b[8];
+        bool pass = true;
 #pragma unroll
-        for (int e = 0; e < 8; ++e) bad |= guard_ok(g_res, acc.y[u][e] + fabsf(x[e]), t[e]) ? 0u : (1u << e);
+        for (int e = 0; e < 8; ++e) {
+            b[e] = fmaf(r, fabsf(x[e]), q * acc.y[u][e]);
+            pass = pass && guard_ok(b[e], t[e]);
+        }
+        unsigned bad = 0;
+        if (!pass)
+#pragma unroll
+            for (int e = 0; e < 8; ++e) bad |= guard_ok(b[e], t[e]) ? 0u : (1u << e);
         while (bad) {
             const int e = __ffs(bad) - 1;
             bad &= bad - 1;

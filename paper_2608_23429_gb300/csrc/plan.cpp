@@ -312,7 +312,8 @@ int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs
         const float hi = on ? (float)w[j] : 0.0f;
         A.w_hi[j] = hi;
         A.w_lo[j] = on ? (float)(w[j] - (double)hi) : 0.0f;
-        A.w_abs[j] = std::fabs(hi);
+        // the fast path's bound, scaled: (K+2) u (1.01) 2^9 |w_hi[j]|, u = 2^-24
+        A.w_guard[j] = (float)(std::fabs((double)hi) * (K + 2) * 1.01 * std::ldexp(1.0, -15));
     }
     A.out_bf16 = out_dtype == CB_BF16;
     A.resid_bf16 = resid_dtype == CB_BF16;
