@@ -6,8 +6,8 @@
  * The method (paper Sec. 3.2-3.3, Alg. 1):
  *   - on full-computation steps s in F, every block's branch outputs f_s are
  *     stored in a history buffer H that holds the n = K most recent
- *     (s_j, f_j) pairs, dropping the oldest (Sec. 3.3, "ChebBooster Forward
- *     Application"; Alg. 1, full-computation branch);
+ *     (s_j, f_j) pairs, dropping the oldest (Sec. 3.3, the forward
+ *     application; Alg. 1, full-computation branch);
  *   - on every other step t the features are predicted as
  *         f_t = sum_j w^j_t f_{s_j}                       (Sec. 3.3, Eq. for f_t)
  *     with the barycentric interpolation coefficients
@@ -95,8 +95,8 @@ enum {
     CB_OPT_PARTIAL_HISTORY = 4 /* 1: while H holds m < K entries (m >= 1), skipped steps use those m
                                   (degree m-1 extrapolation; m = 1 reuses the newest features)
                                   instead of failing with CB_ERR_HISTORY_NOT_FULL. This is Alg. 1
-                                  read literally ("retrieve cached features from H"); default 0,
-                                  the text's reading "provided |H| = n" */
+                                  read literally (extrapolate from whatever H holds); default 0,
+                                  the text's reading (extrapolate only once |H| = n) */
 };
 enum { CB_KERNEL_AUTO = 0, CB_KERNEL_DIRECT = 1, CB_KERNEL_BULK = 2 };
 
@@ -110,7 +110,7 @@ enum {
 /* Full-computation schedule (Sec. 3.3, Eq. for F; Alg. 1 offline stage):
  *   s in F  iff  s not in [s0, T-1-s1]  or  r divides (s - s0),   s in [0, T-1],
  * then, when K > 0, every step whose history would hold fewer than K entries
- * is also marked full (the text's "provided H contains enough entries").
+ * is also marked full (Sec. 3.3 extrapolates only once H holds n entries).
  * is_full: host array of T bytes, written 1 (full) or 0 (extrapolated).
  * n_full: host int, receives the number of full steps (may be NULL).
  * Errors: CB_ERR_ARG for T <= 0, r <= 0, s0 < 0, s1 < 0, K < 0 or is_full NULL. */
@@ -233,7 +233,7 @@ int cb_extrapolate_weights(cb_plan* plan, const double* w_logical, void* const* 
  * CB_OPT_PARTIAL_HISTORY). Errors: CB_ERR_ARG, CB_ERR_HISTORY_NOT_FULL. */
 int cb_weights(const cb_plan* plan, double t_target, double* w_logical);
 
-/* The "prepackaged" weight table (Sec. 3.3; Alg. 1, offline stage): for each
+/* The precomputed weight table (Sec. 3.3; Alg. 1, offline stage): for each
  * targets[m] the weights over the K most recent nodes of node_t that precede
  * it in sampling order, written to table[m*K + j] (j oldest .. newest).
  * Errors: CB_ERR_ARG, CB_ERR_HISTORY_NOT_FULL (fewer than K nodes precede a
@@ -259,8 +259,8 @@ int cb_plan_history(const cb_plan* plan, double* slot_t, int* head, int* count);
 /* Set a plan option (CB_OPT_*). CB_OPT_KERNEL selects the skipped-step
  * kernel: the direct-load kernel (each thread loads its K vectors from HBM) or
  * the bulk-copy pipeline (a producer warp stages the K chunks of each tile in
- * shared memory with cp.async.bulk; CTAs of 544 threads, one per SM); both
- * compute identical bits. CB_OPT_WAIT_NS bounds every wait of the bulk kernel
+ * shared memory with cp.async.bulk; a persistent grid of one or two CTAs per
+ * SM); both compute identical bits. CB_OPT_WAIT_NS bounds every wait of the bulk kernel
  * on a shared-memory barrier; a wait that runs out makes the kernel record a
  * CB_DEV_* code in the device status word and return early (its outputs are
  * then incomplete). Errors: CB_ERR_ARG. */
