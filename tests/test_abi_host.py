@@ -167,7 +167,7 @@ def _workload_nodes(w, orc):
 
 @pytest.mark.parametrize("name", ["dit256", "dit256-k3", "dit512", "pixart", "flux"])
 def test_exported_weight_table_matches_oracle(cb, orc, name):
-    """The prepackaged table (Alg. 1 offline stage) for every skipped step of the
+    """The precomputed weight table (Alg. 1 offline stage) for every skipped step of the
     schedule, against the oracle's Lagrange basis on the same K preceding nodes."""
     from paper_2608_23429_gb300 import workloads
     w = workloads.PRESETS[name]()
