@@ -284,3 +284,43 @@ def test_push_residual(cb, H, src, odd):
             assert st["exact"] >= 0.99 * st["n"], st  # compensated sum: rounded once, like the oracle
     a.close()
     b.close()
+
+
+@pytest.mark.parametrize("layout", ["lone", "groups"])
+def test_maximum_plan(cb, H, layout):
+    """A plan at the ABI's limits: CB_MAX_TENSORS tensors and CB_MAX_K history
+    entries, either 256 lone tensors (256 work items) or 64 residual groups of
+    CB_MAX_BRANCHES members with gated hidden states; both kernels, every
+    element against the oracle."""
+    rng = np.random.default_rng(31)
+    n = cb.CB_MAX_TENSORS
+    tensors = []
+    if layout == "lone":
+        for i in range(n):
+            tensors.append(workloads.TensorSpec(i, 0, (1, int(rng.integers(1, 40)), 64), -1))
+    else:
+        for g in range(n // 4):
+            sh = (int(rng.integers(1, 3)), int(rng.integers(1, 30)), int(rng.choice([64, 40])))
+            tensors += [workloads.TensorSpec(g, m, sh, g) for m in range(4)]
+    K = 8
+    w = workloads.Workload(name=f"max-{layout}", tensors=tensors, K=K, cache_dtype="bf16", T=0, r=0,
+                           t_min=0.0, t_max=999.0, timesteps=[], degree=6, noise=0.1, seed=313)
+    nodes = [990.0 - 30.0 * k for k in range(K)]
+    for kernel in ("bulk", "direct"):
+        walk = H.Walk(w, node_t=nodes, kernel=kernel)
+        cb.cb_plan_set_shapes(walk.plan, [t.shape for t in w.tensors])
+        for k, t in enumerate(nodes):
+            walk.push(t, k)
+        t = nodes[-1] - 20.0
+        if layout == "lone":
+            outs, _, _ = walk.extrapolate(t)
+            so, _, _ = walk.expected_and_compare(t, outs, None, None)
+            _ok(so, (layout, kernel))
+        else:
+            gates = _gates(w, torch.bfloat16, 77)
+            outs, resid, rh = walk.extrapolate(t, fused=True, gates=gates, salt=3)
+            G = [H.expand_gate(g, s.shape) for g, s in zip(gates, w.tensors)]
+            so, sr, _ = walk.expected_and_compare(t, outs, resid, rh, G=G)
+            _ok(so, (layout, kernel, "outs"))
+            _ok(sr, (layout, kernel, "resid"))
+        walk.close()
