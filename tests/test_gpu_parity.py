@@ -479,3 +479,31 @@ def test_bulk_wait_limit_reports_and_recovers(cb, H):
     outs, _, _ = walk.extrapolate(t)
     _assert_ok(walk.expected_and_compare(t, outs, None, None)[0], "after timeout")
     walk.close()
+
+
+def test_element_offsets_beyond_2_31(cb, H):
+    """One tensor of 2^31 + 12345 elements (4.3 GB per slot in bf16, a ragged
+    last tile): the kernels' 64-bit element offsets, checked on sampled
+    elements including both ends and the 2^31 boundary, both kernels."""
+    n = (1 << 31) + 12345
+    w = workloads.Workload(name="huge", tensors=[workloads.TensorSpec(0, 0, (1, 1, n), -1)], K=2,
+                           cache_dtype="bf16", T=0, r=0, t_min=0.0, t_max=999.0, timesteps=[], degree=1,
+                           noise=0.0, seed=71)
+    nodes = [900.0, 850.0]
+    for kernel in ("bulk", "direct"):
+        walk = H.Walk(w, node_t=nodes, kernel=kernel)
+        g = torch.Generator().manual_seed(3)
+        pick = torch.randint(0, n, (4096,), generator=g, dtype=torch.int64)
+        extra = torch.tensor([0, 1, (1 << 31) - 9, (1 << 31) - 1, 1 << 31, (1 << 31) + 7, n - 12345, n - 4096,
+                              n - 1], dtype=torch.int64)
+        walk.idx = [torch.unique(torch.cat([pick, extra])).to("cuda")]
+        for k, t in enumerate(nodes):
+            walk.push(t, k)
+            torch.cuda.empty_cache()
+        outs, _, _ = walk.extrapolate(810.0)
+        so, _, _ = walk.expected_and_compare(810.0, outs, None, None)
+        _assert_ok(so, ("huge", kernel))
+        del outs
+        walk.close()
+        del walk
+        torch.cuda.empty_cache()
