@@ -185,7 +185,10 @@ int push_grid(cb_plan* p, bool sb, bool db, int tiles, int* grid) {
             return cuda_fail(e == cudaSuccess ? cudaErrorInvalidConfiguration : e, "occupancy");
         }
     }
-    long long g = (long long)p->dev.sms * occ;
+    // fewer concurrent copy streams stream faster than full occupancy (FLUX
+    // cache writes: bf16 sources best at 4 CTAs per SM, fp32 sources at 3)
+    const int cap = sb ? 4 : 3;
+    long long g = (long long)p->dev.sms * (occ < cap ? occ : cap);
     *grid = (int)(tiles < g ? tiles : g);
     return CB_OK;
 }
