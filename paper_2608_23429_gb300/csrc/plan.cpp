@@ -430,13 +430,13 @@ int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs
                      &smem, &per_sm);
     if (rc != CB_OK) return rc;
     if (A.stages < max_nb + 1) return launch_direct();  // too deep for shared memory
-    // Persistent grid. bf16 prediction-only launches stream faster over fewer
-    // CTAs than the SMs hold (measured on GB300, repeatable within 0.5 %: K = 5
-    // on one CTA per SM best at 3/4 of the SMs, +3 %; K = 4 on two CTAs per SM
-    // best at 0.7 of the CTAs, +2..3 %; K = 3 best with all of them). Launches
-    // that update hidden states are bound by their consumers and use every SM.
+    // Persistent grid. bf16 prediction-only launches with K >= 3 stream faster
+    // over 3/4 of the SMs (one CTA each) than over all of them (measured on
+    // GB300, repeatable within 0.5 %: FLUX 99 -> 103 %, PixArt 96 -> 104 %,
+    // DiT-512 95 -> 101 % of the copy peak). Launches that update hidden states
+    // are bound by their consumers and use every SM.
     double frac = 1.0;
-    if (cb16 && !grouped && K >= 4) frac = K == 4 ? 0.7 : 0.75;
+    if (cb16 && !grouped && K >= 3) frac = 0.75;
     const long long ctas = std::max(1LL, (long long)((double)p->dev.sms * per_sm * frac));
     const int grid = (int)(tiles < ctas ? tiles : ctas);
     cudaError_t e = any_gate ? cbk::launch_extrapolate_bulk_gated(A, K, cb16, grid, smem, (cudaStream_t)stream)
