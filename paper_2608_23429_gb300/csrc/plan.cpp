@@ -261,18 +261,26 @@ Window live_window(const cb_plan* p, int n) {
 // Gates (one per tensor, [batch, hidden] of gate_dtype, null = 1) apply to the
 // hidden-state update of a grouped tensor: its shape must be set, its group's
 // tensors must share it, and indexing stays in 32 bits.
-int check_gates(const cb_plan* p, void* const* resid, const void* const* gates, cb_dtype gate_dtype) {
+int check_gates(const cb_plan* p, const void* const* gates, cb_dtype gate_dtype) {
     if (!gates) return CB_OK;
     if (!valid_dtype(gate_dtype)) return CB_ERR_ARG;
     const int n = (int)p->tensors.size();
     for (int i = 0; i < n; ++i) {
         if (!gates[i]) continue;
-        const auto& d = p->tensors[i];
         if (p->sh_hidden[i] <= 0) return CB_ERR_ARG;  // cb_plan_set_shapes first
         if (!aligned(gates[i], esize(gate_dtype))) return CB_ERR_ALIGN;
-        if (d.numel > 0xFFFFFFFFLL) return CB_ERR_LIMIT;
-        (void)resid;
+        if (p->tensors[i].numel > 0xFFFFFFFFLL) return CB_ERR_LIMIT;
     }
+    return CB_OK;
+}
+
+// The device status word is zeroed once after binding, on the stream of the
+// first launch, after that launch's arguments have all been validated.
+int clear_status_once(cb_plan* p, void* stream) {
+    if (p->status_clear) return CB_OK;
+    cudaError_t e = cudaMemsetAsync(p->status_word(), 0, sizeof(int), (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
+    p->status_clear = true;
     return CB_OK;
 }
 
@@ -299,7 +307,7 @@ int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs
 
     for (int j = 0; j < K; ++j)
         if (!std::isfinite(w[j])) return CB_ERR_ARG;
-    int rc = check_gates(p, resid, gates, gate_dtype);
+    int rc = check_gates(p, gates, gate_dtype);
     if (rc != CB_OK) return rc;
 
     cbk::ExtrapArgs& A = *p->eargs;
@@ -392,6 +400,8 @@ int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs
         int grid = 0;
         int r = extrap_grid(p, K, cb16, (int)tiles, &grid);
         if (r != CB_OK) return r;
+        r = clear_status_once(p, stream);
+        if (r != CB_OK) return r;
         cudaError_t e = any_gate ? cbk::launch_extrapolate_gated(A, K, cb16, grid, (cudaStream_t)stream)
                                  : cbk::launch_extrapolate(A, K, cb16, grid, (cudaStream_t)stream);
         if (e != cudaSuccess) return cuda_fail(e, "extrapolate launch");
@@ -439,6 +449,8 @@ int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs
     if (cb16 && !grouped && K >= 3) frac = 0.75;
     const long long ctas = std::max(1LL, (long long)((double)p->dev.sms * per_sm * frac));
     const int grid = (int)(tiles < ctas ? tiles : ctas);
+    rc = clear_status_once(p, stream);
+    if (rc != CB_OK) return rc;
     cudaError_t e = any_gate ? cbk::launch_extrapolate_bulk_gated(A, K, cb16, grid, smem, (cudaStream_t)stream)
                              : cbk::launch_extrapolate_bulk(A, K, cb16, grouped, grid, smem, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e, "extrapolate launch");
@@ -544,7 +556,7 @@ int cb_plan_bind_cache(cb_plan* p, void* dev_ptr, size_t bytes) {
     p->cache = static_cast<unsigned char*>(dev_ptr);
     p->next = p->count = 0;
     p->has_last = false;
-    p->status_clear = false;  // zeroed on the stream of the first push
+    p->status_clear = false;  // zeroed on the stream of the first launch
     return CB_OK;
 }
 
@@ -585,13 +597,9 @@ int cb_cache_push(cb_plan* p, const void* const* feats, cb_dtype feat_dtype, dou
     int grid = 0;
     rc = push_grid(p, sb, db, (int)tiles, &grid);
     if (rc != CB_OK) return rc;
-    cudaError_t e;
-    if (!p->status_clear) {
-        e = cudaMemsetAsync(p->status_word(), 0, sizeof(int), (cudaStream_t)stream);
-        if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
-        p->status_clear = true;
-    }
-    e = cbk::launch_push(A, sb, db, grid, (cudaStream_t)stream);
+    rc = clear_status_once(p, stream);
+    if (rc != CB_OK) return rc;
+    cudaError_t e = cbk::launch_push(A, sb, db, grid, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e, "push launch");
     // the pair (t, f_t) is now in H; the oldest entry was overwritten when full
     p->slot_t[p->next] = t;
@@ -687,7 +695,7 @@ int cb_cache_push_residual(cb_plan* p, const void* const* feats, cb_dtype feat_d
     if (resid)
         for (int g = 0; g < ng; ++g)
             if (resid[g] && !aligned(resid[g], res)) return CB_ERR_ALIGN;
-    int rc = check_gates(p, resid, gates, gate_dtype);
+    int rc = check_gates(p, gates, gate_dtype);
     if (rc != CB_OK) return rc;
     if (p->has_last) {
         const double d = t - p->last_t;
@@ -696,13 +704,6 @@ int cb_cache_push_residual(cb_plan* p, const void* const* feats, cb_dtype feat_d
     for (int j = 0; j < p->count; ++j)
         if (p->slot_t[(p->oldest() + j) % p->K] == t) return CB_ERR_NODES_DEGENERATE;
 
-    rc = ensure_device(p);
-    if (rc != CB_OK) return rc;
-    if (!p->status_clear) {
-        cudaError_t e = cudaMemsetAsync(p->status_word(), 0, sizeof(int), (cudaStream_t)stream);
-        if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
-        p->status_clear = true;
-    }
     // one-entry history of weight 1: the new features themselves
     Window one{};
     one.n = 1;
