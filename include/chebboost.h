@@ -52,6 +52,7 @@ extern "C" {
 #define CB_MAX_K 8            /* largest history size n (Sec. 3.3) */
 #define CB_MAX_TENSORS 256    /* branch tensors per plan */
 #define CB_MAX_BRANCHES 4     /* branch tensors sharing one residual group */
+#define CB_MAX_NUMEL (1LL << 48) /* elements per branch tensor */
 #define CB_CACHE_ALIGN 256    /* byte alignment of the cache arena and of each tensor in it */
 #define CB_STATUS_BYTES 256   /* device status block at the end of the cache arena */
 
@@ -81,7 +82,7 @@ enum {
     CB_ERR_ORDER = -5,             /* pushed time does not continue the sampling direction */
     CB_ERR_UNBOUND = -6,           /* no cache arena bound to the plan */
     CB_ERR_CUDA = -7,              /* a CUDA call or launch failed */
-    CB_ERR_LIMIT = -8              /* a size beyond CB_MAX_K / CB_MAX_TENSORS / CB_MAX_BRANCHES */
+    CB_ERR_LIMIT = -8              /* a size beyond one of the CB_MAX_* limits */
 };
 
 /* Options of cb_plan_set_option. */
@@ -124,7 +125,9 @@ int cb_schedule_full(int T, int r, int s0, int s1, int K, uint8_t* is_full, int*
  * tau = 2 (t - t_min) / (t_max - t_min) - 1. tensors: host array of n_tensors
  * descriptors (copied). cache_dtype: storage type of the history buffer.
  * out: receives the new plan. Errors: CB_ERR_ARG (K < 1, n_nodes < K, bad
- * descriptor, t_min >= t_max, non-monotone nodes), CB_ERR_LIMIT,
+ * descriptor, t_min >= t_max, non-monotone nodes), CB_ERR_LIMIT (K >
+ * CB_MAX_K, more than CB_MAX_TENSORS tensors or CB_MAX_BRANCHES members of
+ * a group, a group index >= CB_MAX_TENSORS, numel > CB_MAX_NUMEL),
  * CB_ERR_NODES_DEGENERATE (repeated node time). */
 int cb_plan_create(const double* node_t, int n_nodes, int K, const cb_tensor_desc* tensors,
                    int n_tensors, cb_dtype cache_dtype, double t_min, double t_max, cb_plan** out);

@@ -25,6 +25,7 @@ _lib = ctypes.CDLL(LIB_PATH)
 
 CB_BF16, CB_FP32 = 0, 1
 CB_MAX_K, CB_MAX_TENSORS, CB_MAX_BRANCHES, CB_CACHE_ALIGN, CB_STATUS_BYTES = 8, 256, 4, 256, 256
+CB_MAX_NUMEL = 1 << 48
 CB_OPT_KERNEL, CB_OPT_WAIT_NS, CB_OPT_TEST_WITHHOLD, CB_OPT_PARTIAL_HISTORY = 1, 2, 3, 4
 CB_KERNEL_AUTO, CB_KERNEL_DIRECT, CB_KERNEL_BULK = 0, 1, 2
 CB_DEV_CONSUMER_TIMEOUT, CB_DEV_PRODUCER_TIMEOUT, CB_DEV_DRAIN_TIMEOUT = 1, 2, 4

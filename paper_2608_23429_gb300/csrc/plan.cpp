@@ -510,8 +510,10 @@ int cb_plan_create(const double* node_t, int n_nodes, int K, const cb_tensor_des
         int ng = 0;
         for (const auto& d : p->tensors) {
             if (d.numel <= 0 || d.reserved != 0 || d.group < -1) return CB_ERR_ARG;
+            if (d.numel > CB_MAX_NUMEL) return CB_ERR_LIMIT;
             if (d.group + 1 > ng) ng = d.group + 1;
         }
+        static_assert(cbk::kMaxItems == CB_MAX_TENSORS, "one work item per tensor or group");
         if (ng > cbk::kMaxItems) return CB_ERR_LIMIT;
         p->groups.assign(ng, {});
         for (int i = 0; i < n_tensors; ++i) {
@@ -655,7 +657,10 @@ int cb_plan_set_shapes(cb_plan* p, const int64_t* bth) {
     const int n = (int)p->tensors.size();
     for (int i = 0; i < n; ++i) {
         const int64_t b = bth[3 * i], t = bth[3 * i + 1], h = bth[3 * i + 2];
-        if (b <= 0 || t <= 0 || h <= 0 || b * t * h != p->tensors[i].numel) return CB_ERR_ARG;
+        const int64_t numel = p->tensors[i].numel;
+        // b * t * h == numel, tested by division so that no product overflows
+        if (b <= 0 || t <= 0 || h <= 0 || h > numel || t > numel / h) return CB_ERR_ARG;
+        if (numel % (t * h) != 0 || numel / (t * h) != b) return CB_ERR_ARG;
         if (t * h > 0xFFFFFFFFLL) return CB_ERR_LIMIT;
     }
     for (const auto& g : p->groups)  // members of a group share one hidden state, hence one shape

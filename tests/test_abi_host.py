@@ -37,6 +37,17 @@ def test_every_declared_symbol_is_exported(cb):
     assert set(names) <= set(cb.EXPORTED)
 
 
+def test_constants_match_header(cb):
+    """Every #define and enum value of the header has the same value in the binding."""
+    src = re.sub(r"/\*.*?\*/", "", open(os.path.join(ROOT, "include", "chebboost.h")).read(), flags=re.S)
+    consts = {m[0]: m[1] for m in re.findall(r"#define\s+(CB_\w+)\s+(.+)", src)}
+    consts.update({m[0]: m[1] for m in re.findall(r"\b(CB_\w+)\s*=\s*(-?\d+)", src)})
+    assert len(consts) >= 25
+    for name, text in consts.items():
+        value = eval(text.strip().replace("1LL", "1"), {})
+        assert getattr(cb, name) == value, name
+
+
 def test_status_strings(cb):
     for s in range(0, -9, -1):
         assert cb.cb_status_string(s) and cb.cb_status_string(s) != "unknown status"
@@ -88,6 +99,9 @@ def test_plan_create_errors(cb):
     assert status(tensors=_tensors([8] * 5, [0] * 5)) == cb.CB_ERR_LIMIT  # > CB_MAX_BRANCHES
     assert status(tensors=_tensors([8] * 257)) == cb.CB_ERR_LIMIT
     assert status(tensors=[(0, 0, 8, -2)]) == cb.CB_ERR_ARG
+    assert status(tensors=[(0, 0, 8, cb.CB_MAX_TENSORS)]) == cb.CB_ERR_LIMIT  # group index
+    assert status(tensors=_tensors([cb.CB_MAX_NUMEL])) == 0
+    assert status(tensors=_tensors([8, cb.CB_MAX_NUMEL + 1])) == cb.CB_ERR_LIMIT
 
 
 def test_cache_layout_and_bind(cb):
@@ -217,6 +231,21 @@ def test_shapes_and_gate_validation(cb):
     with pytest.raises(cb.CbError) as e:
         cb.cb_plan_set_shapes(p, [(2, 4, 8), (4, 2, 8), (1, 1, 64)])  # one group, two shapes
     assert e.value.status == cb.CB_ERR_ARG
+    # batch (2^61 + 8) x 8 x 1 wraps to 64 in 64-bit arithmetic: still rejected
+    with pytest.raises(cb.CbError) as e:
+        cb.cb_plan_set_shapes(p, [(2, 4, 8), (2, 4, 8), ((1 << 61) + 8, 8, 1)])
+    assert e.value.status == cb.CB_ERR_ARG
+    for bad in [(0, 8, 8), (1, 1 << 40, 1 << 40), (1, 1, 65), (3, 1, 21)]:
+        with pytest.raises(cb.CbError) as e:
+            cb.cb_plan_set_shapes(p, [(2, 4, 8), (2, 4, 8), bad])
+        assert e.value.status == cb.CB_ERR_ARG, bad
+    with pytest.raises(cb.CbError) as e:  # tokens * hidden >= 2^32
+        big = cb.cb_plan_create([999.0, 900.0], 2, [(0, 0, 1 << 33, -1)], cb.CB_BF16, 0.0, 999.0)
+        try:
+            cb.cb_plan_set_shapes(big, [(1, 1 << 17, 1 << 16)])
+        finally:
+            cb.cb_plan_destroy(big)
+    assert e.value.status == cb.CB_ERR_LIMIT
     cb.cb_plan_bind_cache(p, 0x100000, cb.cb_plan_cache_bytes(p))  # never dereferenced below
     gates = arr(0x3000, 0, 0)
     # history not full is reported before the gates are looked at
