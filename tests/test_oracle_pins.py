@@ -448,6 +448,103 @@ def test_pins_catch_planted_mistakes(orc):
         assert _weight_pins(bad, orc), bad.__name__
 
 
+# ------------------------------------------------------ whole online stage
+def _shifted(s, T=50, a=3.0):
+    """Shifted flow-matching time of step s: t = a u / (1 + (a - 1) u), u = 1 - s/(T-1)."""
+    u = 1.0 - s / (T - 1)
+    return a * u / (1.0 + (a - 1.0) * u)
+
+
+_ONLINE_CASES = [  # (T, r, K, time of step s, t_min, t_max)
+    (50, 4, 3, lambda s: 999.0 * (1 - s / 49), 0.0, 999.0),
+    (50, 5, 4, lambda s: 999.0 * (1 - s / 49), 0.0, 999.0),
+    (20, 3, 4, lambda s: 999.0 * (1 - s / 19), 0.0, 999.0),
+    (50, 6, 5, lambda s: 1.0 - s / 49, 0.0, 1.0),
+    (50, 6, 5, _shifted, 0.0, 1.0),  # non-affine in s
+    (50, 3, 8, lambda s: 999.0 * (1 - s / 49), 0.0, 999.0),
+]
+
+
+def _online_walk(orc, plant=(), seed=31):
+    """Alg. 1's online stage run on the oracle from the schedule to the hidden
+    state, against App. A's error formula. Every element follows a degree-K
+    trajectory F(tau) = sum_{d<=K} c_d T_d(tau) in the normalised time (one
+    degree above what K nodes reproduce). On each skipped step the oracle's
+    prediction must equal F(tau) - c_K 2^(K-1) omega(tau), omega taken over the
+    normalised times of the K most recent full steps, and the hidden state
+    X + sum_b of that.
+    ``plant`` names mistakes planted in copies of the oracle's steps. Returns the
+    largest error relative to its bound (<= 1 passes)."""
+    C = np.polynomial.chebyshev
+    rng = np.random.default_rng(seed)
+    nb, n = 2, 40
+    worst = 0.0
+
+    class Lifo(orc.History):  # planted: drops the newest entry instead of the oldest
+        def push(self, t, f):
+            if self.full():
+                self._h.pop()
+            self._h.append((float(t), f))
+
+    for T, r, K, tf, t_min, t_max in _ONLINE_CASES:
+        c = rng.standard_normal((nb, K + 1, n)) / (1.0 + np.arange(K + 1))[None, :, None]
+        H = Lifo(K) if "lifo" in plant else orc.History(K)
+        mask = orc.full_schedule(T, r, 0, 0, K)
+        assert (~mask).sum() > 0
+        for s in range(T):
+            t = tf(s)
+            tau = 2.0 * (t - t_min) / (t_max - t_min) - 1.0
+            Fs = [C.chebval(tau, c[b]) for b in range(nb)]
+            if mask[s]:
+                H.push(t, Fs)
+                continue
+            times = H.times()
+            w = orc.weights(times, tf(s - 1) if "stale target" in plant else t, t_min, t_max)
+            if "sign" in plant:
+                w[1] = -w[1]
+            if "dropped term" in plant:
+                w[0] = 0.0
+            ent = [f for _, f in H.entries()]
+            if "reversed" in plant:
+                ent = ent[::-1]
+            F = [[e[b] for e in ent] for b in range(nb)]
+            X = rng.standard_normal(n)
+            outs, res = orc.extrapolate(F, w, orc.FP64, orc.FP64, X=X, x_dtype=orc.FP64, resid_dtype=orc.FP64)
+            if "branch missing" in plant:
+                _, res = orc.extrapolate(F[:1], w, orc.FP64, None, X=X, x_dtype=orc.FP64, resid_dtype=orc.FP64)
+            # H holds the K most recent full steps (Sec. 3.3), read off the schedule
+            recent = [tf(q) for q in range(s) if mask[q]][-K:]
+            taus = [2.0 * (x - t_min) / (t_max - t_min) - 1.0 for x in recent]
+            omega = float(np.prod([tau - x for x in taus]))
+            exact_sum = X.copy()
+            bound_sum = 1e-12 * np.abs(X)
+            for b in range(nb):
+                exact = Fs[b] - c[b, K] * 2.0 ** (K - 1) * omega
+                bound = 1e-12 * (np.abs(w) @ np.abs(np.array(F[b])) + np.abs(Fs[b])) + 1e-300
+                worst = max(worst, float(np.max(np.abs(outs[b] - exact) / bound)))
+                exact_sum += exact
+                bound_sum += bound
+            worst = max(worst, float(np.max(np.abs(res - exact_sum) / bound_sum)))
+    return worst
+
+
+def test_online_stage_error_formula(orc):
+    """The oracle's whole online stage on six schedules (DDPM-type, PixArt's
+    T = 20, flow-matching and shifted flow-matching times; K = 3..5 and 8):
+    every skipped step matches App. A's error formula for a degree-K trajectory
+    (which contains the degree <= K-1 exactness of Sec. 3.2 as c_K = 0)."""
+    assert _online_walk(orc) <= 1.0
+
+
+@pytest.mark.parametrize("mistake", ["lifo", "stale target", "sign", "dropped term", "reversed", "branch missing"])
+def test_online_stage_pin_catches_planted_mistakes(orc, mistake):
+    """Mistakes planted on the CPU in copies of the oracle's steps: a history
+    that drops its newest entry, weights for the previous step's time, a
+    flipped weight, a dropped oldest term, weights paired with the history in
+    reverse order, a branch left out of the hidden state."""
+    assert _online_walk(orc, plant=(mistake,)) > 1.0
+
+
 def test_runge_study_report(orc):
     """Sec. 3.2 / Fig. 4: extrapolating f(x) = 1 / (1 + 25 x^2) from K nodes on
     [-1, 1] beyond x = 1 with equispaced nodes, Chebyshev roots, Chebyshev
