@@ -107,6 +107,44 @@ def _ptr_array(xs):
     return ptr_array(xs)
 
 
+# Tensor count, residual-group count and K of every plan this module created:
+# the library reads one pointer per tensor (or group) from each array, so the
+# lengths are checked here before a call.
+_PLANS: dict = {}
+_TENSORS, _GROUPS, _K = 0, 1, 2
+
+
+def _plan_key(plan) -> int | None:
+    return plan.value if isinstance(plan, ctypes.c_void_p) else plan
+
+
+def _dims(plan):
+    return _PLANS.get(_plan_key(plan))
+
+
+def _ptrs(plan, xs, per: int, call: str, what: str):
+    """Pointer array of ``xs`` with one entry per tensor or per residual group."""
+    if xs is None:
+        return None
+    d = _dims(plan)
+    if d is not None and len(xs) != d[per]:
+        unit = "tensors" if per == _TENSORS else "residual groups"
+        raise CbError(CB_ERR_ARG, f"{call} ({what}: {len(xs)} pointers for {d[per]} {unit})")
+    return _ptr_array(xs)
+
+
+def _weights_in(plan, w, call: str):
+    """A caller's weight vector in a CB_MAX_K buffer padded with NaN: the library
+    reads as many entries as the history has live, and rejects non-finite ones."""
+    w = np.ascontiguousarray(w, dtype=np.float64).ravel()
+    d = _dims(plan)
+    if w.size > (d[_K] if d is not None else CB_MAX_K):
+        raise CbError(CB_ERR_ARG, f"{call} ({w.size} weights for K = {d[_K] if d else CB_MAX_K})")
+    buf = np.full(CB_MAX_K, np.nan)
+    buf[:w.size] = w
+    return buf
+
+
 def _stream(s):
     if s is None:
         return None
@@ -135,6 +173,7 @@ def cb_plan_create(node_t, K: int, tensors, cache_dtype: int, t_min: float, t_ma
     _check(_lib.cb_plan_create(node_t.ctypes.data, node_t.size, K, ctypes.cast(descs, ctypes.c_void_p),
                                len(tensors), cache_dtype, float(t_min), float(t_max), ctypes.byref(plan)),
            "cb_plan_create")
+    _PLANS[plan.value] = (len(tensors), int(_lib.cb_plan_num_groups(plan)), int(K))
     return plan
 
 
@@ -147,55 +186,71 @@ def cb_plan_bind_cache(plan, dev_ptr, nbytes: int) -> None:
 
 
 def cb_cache_push(plan, feats, feat_dtype: int, t: float, stream=None) -> None:
-    _check(_lib.cb_cache_push(plan, _ptr_array(feats), feat_dtype, float(t), _stream(stream)), "cb_cache_push")
+    _check(_lib.cb_cache_push(plan, _ptrs(plan, feats, _TENSORS, "cb_cache_push", "feats"), feat_dtype, float(t),
+                              _stream(stream)), "cb_cache_push")
 
 
 def cb_extrapolate(plan, t_target: float, outs, out_dtype: int, resid=None, resid_dtype: int = CB_BF16,
                    stream=None) -> None:
-    _check(_lib.cb_extrapolate(plan, float(t_target), _ptr_array(outs), out_dtype, _ptr_array(resid),
-                               resid_dtype, _stream(stream)), "cb_extrapolate")
+    c = "cb_extrapolate"
+    _check(_lib.cb_extrapolate(plan, float(t_target), _ptrs(plan, outs, _TENSORS, c, "outs"), out_dtype,
+                               _ptrs(plan, resid, _GROUPS, c, "resid"), resid_dtype, _stream(stream)), c)
 
 
 def cb_extrapolate_ring(plan, slot_t, head: int, t_target: float, outs, out_dtype: int, resid=None,
                         resid_dtype: int = CB_BF16, stream=None) -> None:
-    slot_t = _f64(slot_t)
-    _check(_lib.cb_extrapolate_ring(plan, slot_t.ctypes.data, head, float(t_target), _ptr_array(outs),
-                                    out_dtype, _ptr_array(resid), resid_dtype, _stream(stream)),
-           "cb_extrapolate_ring")
+    c = "cb_extrapolate_ring"
+    slot_t = _f64(slot_t).ravel()
+    d = _dims(plan)
+    if d is not None and slot_t.size != d[_K]:  # the library reads K slot times
+        raise CbError(CB_ERR_ARG, f"{c} ({slot_t.size} slot times for K = {d[_K]})")
+    _check(_lib.cb_extrapolate_ring(plan, slot_t.ctypes.data, head, float(t_target),
+                                    _ptrs(plan, outs, _TENSORS, c, "outs"), out_dtype,
+                                    _ptrs(plan, resid, _GROUPS, c, "resid"), resid_dtype, _stream(stream)), c)
 
 
 def cb_extrapolate_weights(plan, w_logical, outs, out_dtype: int, resid=None, resid_dtype: int = CB_BF16,
                            stream=None) -> None:
-    w = _f64(w_logical)
-    _check(_lib.cb_extrapolate_weights(plan, w.ctypes.data, _ptr_array(outs), out_dtype, _ptr_array(resid),
-                                       resid_dtype, _stream(stream)), "cb_extrapolate_weights")
+    c = "cb_extrapolate_weights"
+    w = _weights_in(plan, w_logical, c)
+    _check(_lib.cb_extrapolate_weights(plan, w.ctypes.data, _ptrs(plan, outs, _TENSORS, c, "outs"), out_dtype,
+                                       _ptrs(plan, resid, _GROUPS, c, "resid"), resid_dtype, _stream(stream)), c)
 
 
 def cb_plan_set_shapes(plan, shapes) -> None:
     """``shapes``: sequence of (batch, tokens, hidden), one per tensor."""
-    bth = np.ascontiguousarray(np.asarray(shapes, dtype=np.int64).reshape(-1))
+    bth = np.ascontiguousarray(np.asarray(shapes, dtype=np.int64).reshape(-1, 3))
+    d = _dims(plan)
+    if d is not None and bth.shape[0] != d[_TENSORS]:
+        raise CbError(CB_ERR_ARG, f"cb_plan_set_shapes ({bth.shape[0]} shapes for {d[_TENSORS]} tensors)")
     _check(_lib.cb_plan_set_shapes(plan, bth.ctypes.data), "cb_plan_set_shapes")
 
 
 def cb_extrapolate_gated(plan, t_target: float, outs, out_dtype: int, resid, resid_dtype: int, gates,
                          gate_dtype: int = CB_BF16, stream=None) -> None:
-    _check(_lib.cb_extrapolate_gated(plan, float(t_target), _ptr_array(outs), out_dtype, _ptr_array(resid),
-                                     resid_dtype, _ptr_array(gates), gate_dtype, _stream(stream)),
-           "cb_extrapolate_gated")
+    c = "cb_extrapolate_gated"
+    _check(_lib.cb_extrapolate_gated(plan, float(t_target), _ptrs(plan, outs, _TENSORS, c, "outs"), out_dtype,
+                                     _ptrs(plan, resid, _GROUPS, c, "resid"), resid_dtype,
+                                     _ptrs(plan, gates, _TENSORS, c, "gates"), gate_dtype, _stream(stream)), c)
 
 
 def cb_cache_push_residual(plan, feats, feat_dtype: int, t: float, resid, resid_dtype: int = CB_BF16,
                            gates=None, gate_dtype: int = CB_BF16, stream=None) -> None:
-    _check(_lib.cb_cache_push_residual(plan, _ptr_array(feats), feat_dtype, float(t), _ptr_array(resid),
-                                       resid_dtype, _ptr_array(gates), gate_dtype, _stream(stream)),
-           "cb_cache_push_residual")
+    c = "cb_cache_push_residual"
+    _check(_lib.cb_cache_push_residual(plan, _ptrs(plan, feats, _TENSORS, c, "feats"), feat_dtype, float(t),
+                                       _ptrs(plan, resid, _GROUPS, c, "resid"), resid_dtype,
+                                       _ptrs(plan, gates, _TENSORS, c, "gates"), gate_dtype, _stream(stream)), c)
 
 
 def cb_weights(plan, t_target: float, n: int) -> np.ndarray:
-    """Weights over the n live history entries (n = K, or fewer under partial history)."""
-    w = np.empty(n, dtype=np.float64)
+    """Weights over the n live history entries (n = K, or fewer under partial history).
+    The library writes one weight per live entry into a CB_MAX_K buffer; entries
+    beyond them stay NaN."""
+    if not 1 <= n <= CB_MAX_K:
+        raise CbError(CB_ERR_ARG, f"cb_weights (n = {n})")
+    w = np.full(CB_MAX_K, np.nan)
     _check(_lib.cb_weights(plan, float(t_target), w.ctypes.data), "cb_weights")
-    return w
+    return w[:n].copy()
 
 
 def cb_taylor_weights(node_t, t_target: float) -> np.ndarray:
@@ -207,7 +262,11 @@ def cb_taylor_weights(node_t, t_target: float) -> np.ndarray:
 
 
 def cb_plan_export_weights(plan, targets, K: int) -> np.ndarray:
+    """One row of the plan's K weights per target (the library writes rows of K)."""
     targets = _f64(targets)
+    d = _dims(plan)
+    if (d is not None and K != d[_K]) or not 1 <= K <= CB_MAX_K:
+        raise CbError(CB_ERR_ARG, f"cb_plan_export_weights (K = {K})")
     table = np.empty((targets.size, K), dtype=np.float64)
     _check(_lib.cb_plan_export_weights(plan, targets.ctypes.data, targets.size, table.ctypes.data),
            "cb_plan_export_weights")
@@ -215,6 +274,10 @@ def cb_plan_export_weights(plan, targets, K: int) -> np.ndarray:
 
 
 def cb_plan_history(plan, K: int):
+    """Slot times (the library writes the plan's K of them), oldest slot, count."""
+    d = _dims(plan)
+    if (d is not None and K != d[_K]) or not 1 <= K <= CB_MAX_K:
+        raise CbError(CB_ERR_ARG, f"cb_plan_history (K = {K})")
     slot_t = np.empty(K, dtype=np.float64)
     head, count = ctypes.c_int(0), ctypes.c_int(0)
     _check(_lib.cb_plan_history(plan, slot_t.ctypes.data, ctypes.byref(head), ctypes.byref(count)),
@@ -241,6 +304,7 @@ def cb_plan_num_groups(plan) -> int:
 
 
 def cb_plan_destroy(plan) -> None:
+    _PLANS.pop(_plan_key(plan), None)
     _lib.cb_plan_destroy(plan)
 
 

@@ -260,3 +260,46 @@ def test_shapes_and_gate_validation(cb):
     assert st("cb_cache_push_residual", p, feats, 0, 999.0, arr(0x5001), 0, gates, 0, None) == cb.CB_ERR_ALIGN
     assert st("cb_cache_push_residual", p, feats, 0, 999.0, arr(0x5000), 0, gates, 9, None) == cb.CB_ERR_ARG
     cb.cb_plan_destroy(p)
+
+
+def test_binding_checks_array_lengths(cb):
+    """The binding refuses pointer lists, shapes, slot times and weight vectors
+    whose length does not match the plan before the library reads them."""
+    p = cb.cb_plan_create([999.0, 900.0, 800.0], 3, [(0, 0, 64, 0), (0, 1, 64, 0), (1, 0, 32, -1)],
+                          cb.CB_BF16, 0.0, 999.0)
+    two, three = [0x1000, 0x2000], [0x1000, 0x2000, 0x3000]
+    calls = [
+        lambda: cb.cb_cache_push(p, two, cb.CB_BF16, 999.0),
+        lambda: cb.cb_extrapolate(p, 700.0, two, cb.CB_BF16),
+        lambda: cb.cb_extrapolate(p, 700.0, three, cb.CB_BF16, resid=two),  # one residual group
+        lambda: cb.cb_extrapolate_ring(p, [999.0, 900.0], 0, 700.0, three, cb.CB_BF16),
+        lambda: cb.cb_extrapolate_weights(p, [0.1, 0.2, 0.3, 0.4], three, cb.CB_BF16),
+        lambda: cb.cb_extrapolate_gated(p, 700.0, three, cb.CB_BF16, [0x5000], cb.CB_BF16, two),
+        lambda: cb.cb_cache_push_residual(p, two, cb.CB_BF16, 999.0, [0x5000]),
+        lambda: cb.cb_cache_push_residual(p, three, cb.CB_BF16, 999.0, two),
+        lambda: cb.cb_plan_set_shapes(p, [(1, 8, 8), (1, 8, 8)]),
+        lambda: cb.cb_weights(p, 700.0, 9),
+        lambda: cb.cb_plan_export_weights(p, [700.0], 2),
+        lambda: cb.cb_plan_history(p, 2),
+    ]
+    for i, call in enumerate(calls):
+        with pytest.raises(cb.CbError) as e:
+            call()
+        assert e.value.status == cb.CB_ERR_ARG, i
+    # lengths that match reach the library (which reports its own status)
+    with pytest.raises(cb.CbError) as e:
+        cb.cb_extrapolate(p, 700.0, three, cb.CB_BF16, resid=[0x5000])
+    assert e.value.status == cb.CB_ERR_UNBOUND
+    assert len(cb.cb_plan_history(p, 3)[0]) == 3
+    cb.cb_plan_destroy(p)
+
+
+def test_short_weight_vector_is_rejected_not_overread(cb):
+    """cb_extrapolate_weights reads one weight per live entry: a shorter vector
+    reaches the library padded with NaN and is refused as non-finite."""
+    p = cb.cb_plan_create([999.0, 900.0], 2, [(0, 0, 64, -1)], cb.CB_BF16, 0.0, 999.0)
+    cb.cb_plan_set_option(p, cb.CB_OPT_PARTIAL_HISTORY, 1)
+    buf = cb._weights_in(p, [0.5], "test")
+    assert buf.size == cb.CB_MAX_K and buf[0] == 0.5 and np.isnan(buf[1:]).all()
+    cb.cb_plan_destroy(p)
+    assert cb._dims(p) is None
