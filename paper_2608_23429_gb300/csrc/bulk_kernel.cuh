@@ -12,12 +12,13 @@
 // consumers' registers, which is what bounds the direct-load variant.
 //
 // Many consumer warps per scheduler hide the consumers' fixed latencies (see
-// Shape for the thread map). Two kinds of launch (GROUPED):
-//   * predictions only: each stage is released as soon as it is in
-//     registers, and guarded elements are recomputed from registers;
-//   * with hidden states: stages are released after the member's arithmetic,
-//     guarded elements are recomputed from shared memory (so the history
-//     values die early). The producer also stages each tile's bf16 hidden
+// Shape for the thread map). A stage goes back to the producer only after the
+// arithmetic has used every value read from it (release_stage). Two kinds of
+// launch (GROUPED):
+//   * predictions only: guarded elements are recomputed from the registers
+//     the history values were loaded into;
+//   * with hidden states: guarded elements are recomputed from shared memory
+//     (so the history values die early). The producer also stages each tile's bf16 hidden
 //     state (one more chunk with the group's last member) and the consumers
 //     hold the group's member stages until the hidden state is written (the
 //     host guarantees more stages than members, so holding cannot starve the
@@ -28,8 +29,10 @@
 // one-entry history of weight 1 whose member addresses are the new features;
 // with copy_out the outputs (the ring slot) receive the features converted.
 //
-// Every wait is bounded (%globaltimer). A wait that runs out records a code in
-// the plan's device status word and the thread returns; the producer then
+// Every wait is bounded (%globaltimer). A consumer wait that runs out in any
+// lane records a code in the plan's device status word and the whole warp
+// returns (a warp vote, so no lane leaves a warp that goes on to a
+// __syncwarp); a producer wait that runs out stops the producer, which then
 // waits, with its own limit (at least 10 ms), for the copies it has issued
 // before it exits. A test option makes the producer announce the first unit's
 // bytes without issuing its copies, so that the consumers' wait runs out with
@@ -116,6 +119,25 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t
 
 __device__ __forceinline__ void record(int* status, int code) {
     if (status) atomicOr(status, code);
+}
+
+// Orders this thread's earlier generic-proxy accesses of shared memory before
+// later async-proxy accesses (the bulk copies that refill a released stage).
+__device__ __forceinline__ void fence_generic_to_async() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// A consumer warp hands one stage back to the producer. It is called only
+// after the values the warp read from the stage have been used (stored or
+// accumulated), so every shared-memory load of the stage has returned; each
+// lane then fences its reads against the async proxy before lane 0 arrives.
+// Releasing right after issuing the loads, with the loaded values still unused,
+// let a refill land on the start of the stage before a warp's loads were
+// performed (half a warp's first vector read the next unit's bytes).
+__device__ __forceinline__ void release_stage(uint32_t empty_bar, int lane) {
+    fence_generic_to_async();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(empty_bar);
 }
 
 // GROUPED: some item updates a hidden state or has several members (stage
@@ -264,8 +286,10 @@ __global__ void __launch_bounds__(Shape<CB16, K, GROUPED, GATED>::threads, Shape
         acc.zero();
         for (int m = 0; m < nb; ++m) {
             const uint32_t stage = cs;
-            if (!mbar_wait(full0 + 8u * stage, cph, A.wait_ns)) {
-                record(A.status, 1);
+            // the give-up is warp-uniform: no lane leaves while its warp-mates
+            // go on to a __syncwarp
+            if (!__all_sync(~0u, mbar_wait(full0 + 8u * stage, cph, A.wait_ns))) {
+                if (lane == 0) record(A.status, 1);
                 return;
             }
             if (++cs == (uint32_t)S) {
@@ -294,14 +318,11 @@ __global__ void __launch_bounds__(Shape<CB16, K, GROUPED, GATED>::threads, Shape
 #pragma unroll
                     for (int e = 0; e < 8; ++e) gv[e] = 1.0f;
             };
-            // prediction-only launches release the stage at once and recompute
-            // guarded elements from registers; grouped launches keep the stage
-            // until the member is done and recompute from shared memory, which
-            // frees the history values' registers early
-            if (!GROUPED) {
-                __syncwarp();
-                if (lane == 0) mbar_arrive(empty0 + 8u * stage);
-            }
+            // prediction-only launches recompute guarded elements from the
+            // registers; grouped launches recompute from shared memory, which
+            // frees the history values' registers early. Either way the stage is
+            // released only after the arithmetic has consumed what was read
+            // from it (release_stage).
             if (full_tile && mine) {
                 void* out = member_out<K, CB16, U>(A, first + m, ev, raw);
                 if (A.precise) {
@@ -326,10 +347,7 @@ __global__ void __launch_bounds__(Shape<CB16, K, GROUPED, GATED>::threads, Shape
                                                          acc, gate);
                 }
             }
-            if (GROUPED && !hold) {
-                __syncwarp();
-                if (lane == 0) mbar_arrive(empty0 + 8u * stage);
-            }
+            if (!hold) release_stage(empty0 + 8u * stage, lane);
         }
         if (GROUPED && hold) {
             const uint32_t last = stage_of(nb - 1);
@@ -373,6 +391,7 @@ __global__ void __launch_bounds__(Shape<CB16, K, GROUPED, GATED>::threads, Shape
                 };
                 resid_fast<K, U>(A, it, ev, acc, resid, xload, exact);
             }
+            fence_generic_to_async();
             __syncwarp();
             if (lane == 0)
                 for (int m = 0; m < nb; ++m) mbar_arrive(empty0 + 8u * stage_of(m));

@@ -158,6 +158,88 @@ def test_pixart_scaled_outputs_and_fp32(cb, H):
     walk.close()
 
 
+# ------------------------------------- repeated launches give the same bits
+def _launch(cb, H, walk, t, kernel, resid0=None):
+    """One skipped step into output buffers filled with NaN (an element the
+    kernel fails to write cannot pass as a stale copy of an earlier launch);
+    with resid0 the hidden states start from a copy of those tensors."""
+    cb.cb_plan_set_option(walk.plan, cb.CB_OPT_KERNEL, H.KERNEL[kernel])
+    outs = [torch.full(s.shape, float("nan"), dtype=torch.bfloat16, device="cuda") for s in walk.w.tensors]
+    resid = None if resid0 is None else [r.clone() for r in resid0]
+    cb.cb_extrapolate(walk.plan, t, outs, cb.CB_BF16, resid, cb.CB_BF16)
+    torch.cuda.synchronize()
+    assert cb.cb_plan_device_status(walk.plan) == 0
+    return outs + (resid or [])
+
+
+def _same_bits(a, b):
+    return sum(int((x.view(torch.int16) != y.view(torch.int16)).sum()) for x, y in zip(a, b))
+
+
+def _repeat(cb, H, walk, t, reps, fused=False, salt=0):
+    """The oracle checks the first bulk launch; every further launch, and the
+    direct kernel's, must write exactly the same bits."""
+    resid0 = None
+    rh = None
+    if fused:
+        resid0 = [workloads.hidden_state(walk.w, g, "cuda", salt=salt) for g in range(walk.n_groups)]
+        rh = [H.host(resid0[g], walk._gidx(g)) for g in range(walk.n_groups)]
+    first = _launch(cb, H, walk, t, "bulk", resid0)
+    nt = len(walk.w.tensors)
+    so, sr, _ = walk.expected_and_compare(t, first[:nt], first[nt:] if fused else None, rh)
+    _assert_ok(so, ("repeat: first launch", t))
+    if fused:
+        _assert_ok(sr, ("repeat: first launch, hidden states", t))
+    assert _same_bits(first, _launch(cb, H, walk, t, "direct", resid0)) == 0, "direct kernel differs"
+    diffs = [_same_bits(first, _launch(cb, H, walk, t, "bulk", resid0)) for _ in range(reps)]
+    assert not any(diffs), diffs
+    cb.cb_plan_set_option(walk.plan, cb.CB_OPT_KERNEL, H.KERNEL["auto"])
+
+
+def test_repeat_partial_history_step(cb, H):
+    """PixArt/32 with no warm-up full steps, n = 2 live entries at step 5: a
+    prediction-only launch of two CTAs per SM, 20 times over."""
+    w = workloads.scaled(workloads.pixart(), 32)
+    mask = H.library_schedule(w, 0)
+    node_t = [t for s, t in enumerate(w.timesteps) if mask[s]]
+    walk = H.Walk(w, node_t=node_t)
+    cb.cb_plan_set_option(walk.plan, cb.CB_OPT_PARTIAL_HISTORY, 1)
+    walk.push(w.timesteps[0], 0)
+    walk.push(w.timesteps[3], 3)
+    _repeat(cb, H, walk, w.timesteps[5], 20)
+    walk.close()
+
+
+@pytest.mark.parametrize("K", range(1, 9))
+def test_repeat_prediction_only_shapes(cb, H, K):
+    """Every prediction-only launch shape (K = 1..8) on PixArt/4 (48384 tiles,
+    so every CTA cycles its stage ring many times), 20 launches each."""
+    w = workloads.scaled(workloads.pixart(), 4)
+    nodes = [999.0 - 45.0 * k for k in range(K)]
+    walk = H.Walk(w, K=K, node_t=nodes, samples=4096, seed=K)
+    for k, t in enumerate(nodes):
+        walk.push(t, k)
+    _repeat(cb, H, walk, nodes[-1] - 30.0, 20)
+    walk.close()
+    torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("K,fused", [(1, False), (2, False), (3, True)])
+def test_repeat_full_size_two_ctas_per_sm(cb, H, K, fused):
+    """Full-size PixArt-Sigma 1024^2 shapes in the launches that run two CTAs
+    per SM (K = 1 and 2 prediction-only; K = 3 with the hidden states fused),
+    20 launches each."""
+    w = workloads.pixart()
+    nodes = [999.0 - 45.0 * k for k in range(K)]
+    walk = H.Walk(w, K=K, node_t=nodes, samples=2048, seed=10 + K)
+    for k, t in enumerate(nodes):
+        walk.push(t, k)
+        torch.cuda.empty_cache()
+    _repeat(cb, H, walk, nodes[-1] - 30.0, 20, fused=fused, salt=K)
+    walk.close()
+    torch.cuda.empty_cache()
+
+
 # --------------------------------------------- full-size, sampled outputs
 FULL = {
     "dit256": (lambda: workloads.dit256(4), True),
