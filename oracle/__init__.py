@@ -11,7 +11,9 @@ oldest entry is dropped when it is full (Sec. 3.3).
 from __future__ import annotations
 
 import ctypes
+import hashlib
 import os
+import platform
 import subprocess
 from collections import deque
 
@@ -27,14 +29,29 @@ _NP = {BF16: np.uint16, FP32: np.float32, FP64: np.float64}
 _lib = None
 
 
+_CFLAGS = ["-O2", "-std=c11", "-fPIC", "-shared", "-fno-fast-math", "-ffp-contract=off"]
+_STAMP = os.path.join(_HERE, "liborc.stamp")
+
+
+def _stamp() -> str:
+    with open(_SRC, "rb") as fh:
+        h = hashlib.sha256(fh.read())
+    h.update(" ".join(_CFLAGS).encode())
+    h.update(platform.machine().encode())
+    return h.hexdigest()
+
+
 def build(force: bool = False) -> str:
-    """Compile the oracle with gcc into ``oracle/liborc.so`` (idempotent)."""
-    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+    """Compile the oracle with gcc into ``oracle/liborc.so``; an existing build is
+    reused only when its stamp (source, flags, machine) matches."""
+    stamp = _stamp()
+    current = os.path.exists(_LIB) and os.path.exists(_STAMP) and open(_STAMP).read().strip() == stamp
+    if force or not current:
         tmp = _LIB + f".tmp{os.getpid()}"
-        subprocess.check_call(
-            ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fno-fast-math", "-ffp-contract=off",
-             "-o", tmp, _SRC, "-lm", "-lpthread"])
+        subprocess.check_call(["gcc", *_CFLAGS, "-o", tmp, _SRC, "-lm", "-lpthread"])
         os.replace(tmp, _LIB)
+        with open(_STAMP, "w") as fh:
+            fh.write(stamp + "\n")
     return _LIB
 
 
