@@ -5,7 +5,7 @@ caches, aligned and ragged hidden sizes, lone tensors and residual groups of
 read from global memory, partial history, both kernels), each compared with
 the oracle element by element (Sec. 3.3, Eq. for f_t; Sec. 3.1 residual).
 
-Same gates as test_gpu_parity.py: bf16 within one ulp of the oracle's fp64
+Same gates as test_gpu_a_parity.py: bf16 within one ulp of the oracle's fp64
 result rounded to bf16 (exact cancellations below 2^-40 sum|w F| counted
 apart), fp32 within 2e-6 max|F|.
 """

@@ -1,7 +1,7 @@
 """GPU parity for the widened rows: partial history during warm-up, caller-given
 weights (other node families, truncated Taylor), and a non-affine schedule.
 
-Same gates as test_gpu_parity.py: within one bf16 ulp of the oracle's fp64
+Same gates as test_gpu_a_parity.py: within one bf16 ulp of the oracle's fp64
 result rounded to bf16 (exact cancellations below 2^-40 sum|w F| counted apart).
 """
 import numpy as np
@@ -40,7 +40,7 @@ def test_partial_history_warmup(cb, H, kernel):
     """Alg. 1 read literally: with no warm-up full steps, the steps after the
     first full step extrapolate from the 1, 2, ... entries H holds."""
     w = workloads.scaled(workloads.pixart(), 32)
-    mask = orc.full_schedule(w.T, w.r, 0, 0, 0)  # the set F alone
+    mask = H.library_schedule(w, 0)  # the set F alone (no warm-up rule)
     node_t = [t for s, t in enumerate(w.timesteps) if mask[s]]
     walk = H.Walk(w, node_t=node_t, kernel=kernel)
     walk.push(w.timesteps[0], 0)
@@ -57,6 +57,13 @@ def test_partial_history_warmup(cb, H, kernel):
         n = len(walk.H.entries())
         used.add(n)
         wl = cb.cb_weights(walk.plan, t, n)
+        if n < w.K:  # a count other than the live entries' is refused, not truncated or padded
+            for call in (lambda: cb.cb_weights(walk.plan, t, n + 1),
+                         lambda: cb.cb_extrapolate_weights(walk.plan, np.full(n + 1, 1.0 / (n + 1)), None,
+                                                           cb.CB_BF16)):
+                with pytest.raises(cb.CbError) as e:
+                    call()
+                assert e.value.status == cb.CB_ERR_ARG
         ref = orc.weights(walk.H.times(), t, w.t_min, w.t_max)
         assert np.max(np.abs(wl - ref)) <= 1e-12 * np.abs(ref).sum()
         outs, resid, rh = walk.extrapolate(t, fused=(s % 2 == 0), salt=s)
@@ -161,7 +168,7 @@ def test_gated_residual(cb, H, kernel, resid_dtype):
 
 def test_gated_residual_odd_shapes(cb, H):
     """Hidden sizes that are not multiples of 8 (scalar path), fp32 gates."""
-    from test_gpu_parity import _odd_workload
+    from test_gpu_a_parity import _odd_workload
     w = _odd_workload(4)
     nodes = [950.0, 900.0, 850.0, 800.0]
     walk = H.Walk(w, node_t=nodes)
@@ -248,7 +255,7 @@ def test_push_residual(cb, H, src, odd):
     """Full step with the fused epilogue: the slots hold exactly what the plain
     push writes, and x <- x + sum_b g_b f_b (un-rounded features) matches the
     oracle's single rounding."""
-    from test_gpu_parity import _odd_workload
+    from test_gpu_a_parity import _odd_workload
     w = _odd_workload(3) if odd else workloads.scaled(workloads.pixart(), 32)
     w.cache_dtype = "bf16"
     nodes = [900.0, 800.0, 700.0]
