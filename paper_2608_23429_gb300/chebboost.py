@@ -107,11 +107,12 @@ def _ptr_array(xs):
     return ptr_array(xs)
 
 
-# Tensor count, residual-group count and K of every plan this module created:
-# the library reads one pointer per tensor (or group) from each array, so the
-# lengths are checked here before a call.
+# Tensor count, residual-group count, K and the partial-history option of every
+# plan this module created: the library reads one pointer per tensor (or group)
+# from each array and one weight per live history entry, so the lengths are
+# checked here before a call.
 _PLANS: dict = {}
-_TENSORS, _GROUPS, _K = 0, 1, 2
+_TENSORS, _GROUPS, _K, _PARTIAL = 0, 1, 2, 3
 
 
 def _plan_key(plan) -> int | None:
@@ -133,13 +134,30 @@ def _ptrs(plan, xs, per: int, call: str, what: str):
     return _ptr_array(xs)
 
 
+def _live(plan) -> int | None:
+    """History entries a skipped step of this plan uses now: K once H is full,
+    what H holds under the partial-history option, else 0 (the library then
+    reports the history as not full). None for a plan made elsewhere."""
+    d = _dims(plan)
+    if d is None:
+        return None
+    count = ctypes.c_int(0)
+    _check(_lib.cb_plan_history(plan, None, None, ctypes.byref(count)), "cb_plan_history")
+    if count.value >= d[_K]:
+        return d[_K]
+    return count.value if d[_PARTIAL] else 0
+
+
 def _weights_in(plan, w, call: str):
     """A caller's weight vector in a CB_MAX_K buffer padded with NaN: the library
-    reads as many entries as the history has live, and rejects non-finite ones."""
+    reads one entry per live history entry and rejects non-finite ones, so a
+    vector of any other length is refused here."""
     w = np.ascontiguousarray(w, dtype=np.float64).ravel()
     d = _dims(plan)
-    if w.size > (d[_K] if d is not None else CB_MAX_K):
-        raise CbError(CB_ERR_ARG, f"{call} ({w.size} weights for K = {d[_K] if d else CB_MAX_K})")
+    live = _live(plan)
+    if w.size > (d[_K] if d is not None else CB_MAX_K) or (live and w.size != live):
+        raise CbError(CB_ERR_ARG, f"{call} ({w.size} weights for {live} live history entries, "
+                                  f"K = {d[_K] if d is not None else '?'})")
     buf = np.full(CB_MAX_K, np.nan)
     buf[:w.size] = w
     return buf
@@ -173,7 +191,7 @@ def cb_plan_create(node_t, K: int, tensors, cache_dtype: int, t_min: float, t_ma
     _check(_lib.cb_plan_create(node_t.ctypes.data, node_t.size, K, ctypes.cast(descs, ctypes.c_void_p),
                                len(tensors), cache_dtype, float(t_min), float(t_max), ctypes.byref(plan)),
            "cb_plan_create")
-    _PLANS[plan.value] = (len(tensors), int(_lib.cb_plan_num_groups(plan)), int(K))
+    _PLANS[plan.value] = [len(tensors), int(_lib.cb_plan_num_groups(plan)), int(K), False]
     return plan
 
 
@@ -242,15 +260,18 @@ def cb_cache_push_residual(plan, feats, feat_dtype: int, t: float, resid, resid_
                                        _ptrs(plan, gates, _TENSORS, c, "gates"), gate_dtype, _stream(stream)), c)
 
 
-def cb_weights(plan, t_target: float, n: int) -> np.ndarray:
-    """Weights over the n live history entries (n = K, or fewer under partial history).
-    The library writes one weight per live entry into a CB_MAX_K buffer; entries
-    beyond them stay NaN."""
-    if not 1 <= n <= CB_MAX_K:
-        raise CbError(CB_ERR_ARG, f"cb_weights (n = {n})")
+def cb_weights(plan, t_target: float, n: int | None = None) -> np.ndarray:
+    """Weights over the live history entries (K, or fewer under partial history),
+    oldest first. ``n``, if given, must equal that count. The library writes one
+    weight per live entry into a CB_MAX_K buffer."""
+    live = _live(plan)
+    if n is not None and (not 1 <= n <= CB_MAX_K or (live and n != live)):
+        raise CbError(CB_ERR_ARG, f"cb_weights (n = {n} for {live} live history entries)")
     w = np.full(CB_MAX_K, np.nan)
     _check(_lib.cb_weights(plan, float(t_target), w.ctypes.data), "cb_weights")
-    return w[:n].copy()
+    if live is None:
+        live = n if n is not None else int(np.isfinite(w).sum())
+    return w[:live].copy()
 
 
 def cb_taylor_weights(node_t, t_target: float) -> np.ndarray:
@@ -291,6 +312,9 @@ def cb_plan_reset(plan) -> None:
 
 def cb_plan_set_option(plan, option: int, value: int) -> None:
     _check(_lib.cb_plan_set_option(plan, option, int(value)), "cb_plan_set_option")
+    d = _dims(plan)
+    if d is not None and option == CB_OPT_PARTIAL_HISTORY:
+        d[_PARTIAL] = bool(value)
 
 
 def cb_plan_device_status(plan, stream=None) -> int:

@@ -86,7 +86,7 @@ class Walk:
         self.dev = torch.device(device)
         self.cdt = w.cache_dtype
         if node_t is None:
-            self.full = orc.full_schedule(w.T, w.r, w.s0, w.s1, self.K)
+            self.full = library_schedule(w, self.K)
             node_t = [t for s, t in enumerate(w.timesteps) if self.full[s]]
         self.node_t = list(node_t)
         self.tensors = [(t.layer, t.branch, t.numel, t.group) for t in w.tensors]
@@ -206,8 +206,16 @@ class Walk:
         return merge(stats_out) if stats_out else None, merge(stats_res) if stats_res else None, wts
 
 
+def library_schedule(w: workloads.Workload, K: int) -> np.ndarray:
+    """The full-step mask the product drives its runs with (the library's
+    cb_schedule_full), checked here against the oracle's own schedule."""
+    mask, _ = cb.cb_schedule_full(w.T, w.r, w.s0, w.s1, K)
+    assert np.array_equal(mask, orc.full_schedule(w.T, w.r, w.s0, w.s1, K)), (w.name, K)
+    return mask
+
+
 def schedule_steps(w: workloads.Workload, K: int):
-    mask = orc.full_schedule(w.T, w.r, w.s0, w.s1, K)
+    mask = library_schedule(w, K)
     return mask, [s for s in range(w.T) if not mask[s]]
 
 

@@ -174,7 +174,9 @@ def test_failed_launch_leaves_history_unchanged(cb):
 
 
 def _workload_nodes(w, orc):
-    mask = orc.full_schedule(w.T, w.r, w.s0, w.s1, w.K)
+    from paper_2608_23429_gb300 import chebboost as cb
+    mask, _ = cb.cb_schedule_full(w.T, w.r, w.s0, w.s1, w.K)  # the product's schedule
+    assert np.array_equal(mask, orc.full_schedule(w.T, w.r, w.s0, w.s1, w.K))
     ts = np.array(w.timesteps)
     return ts[mask], ts[~mask]
 
