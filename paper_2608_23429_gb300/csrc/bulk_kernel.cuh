@@ -12,13 +12,14 @@
 // consumers' registers, which is what bounds the direct-load variant.
 //
 // Many consumer warps per scheduler hide the consumers' fixed latencies (see
-// Shape for the thread map). A stage goes back to the producer only after the
-// arithmetic has used every value read from it (release_stage). Two kinds of
-// launch (GROUPED):
-//   * predictions only: guarded elements are recomputed from the registers
-//     the history values were loaded into;
-//   * with hidden states: guarded elements are recomputed from shared memory
-//     (so the history values die early). The producer also stages each tile's bf16 hidden
+// Shape for the thread map). Every consumer fences its reads of a stage
+// against the async proxy before the stage goes back to the producer
+// (release_stage). Two kinds of launch (GROUPED):
+//   * predictions only: each stage is released as soon as it is read into
+//     registers, and guarded elements are recomputed from those registers;
+//   * with hidden states: stages are released after the member's arithmetic,
+//     guarded elements are recomputed from shared memory (so the history
+//     values die early). The producer also stages each tile's bf16 hidden
 //     state (one more chunk with the group's last member) and the consumers
 //     hold the group's member stages until the hidden state is written (the
 //     host guarantees more stages than members, so holding cannot starve the
@@ -127,13 +128,14 @@ __device__ __forceinline__ void fence_generic_to_async() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
-// A consumer warp hands one stage back to the producer. It is called only
-// after the values the warp read from the stage have been used (stored or
-// accumulated), so every shared-memory load of the stage has returned; each
-// lane then fences its reads against the async proxy before lane 0 arrives.
-// Releasing right after issuing the loads, with the loaded values still unused,
-// let a refill land on the start of the stage before a warp's loads were
-// performed (half a warp's first vector read the next unit's bytes).
+// A consumer warp hands one stage back to the producer: every lane fences its
+// shared-memory reads of the stage against the async proxy, then lane 0
+// arrives on the stage's empty barrier. The refill that follows is an
+// async-proxy write to the same bytes, and the mbarrier release/acquire pair
+// alone does not order it after generic-proxy reads: without the fence, a
+// refill landed on the start of a stage before some of a warp's loads were
+// performed (half a warp's first vector took the next unit's bytes, about one
+// launch in 200 on full-size PixArt shapes; none in 3000 with the fence).
 __device__ __forceinline__ void release_stage(uint32_t empty_bar, int lane) {
     fence_generic_to_async();
     __syncwarp();
@@ -318,11 +320,11 @@ __global__ void __launch_bounds__(Shape<CB16, K, GROUPED, GATED>::threads, Shape
 #pragma unroll
                     for (int e = 0; e < 8; ++e) gv[e] = 1.0f;
             };
-            // prediction-only launches recompute guarded elements from the
-            // registers; grouped launches recompute from shared memory, which
-            // frees the history values' registers early. Either way the stage is
-            // released only after the arithmetic has consumed what was read
-            // from it (release_stage).
+            // prediction-only launches release the stage as soon as it is read
+            // and recompute guarded elements from registers; grouped launches
+            // keep the stage until the member is done and recompute from shared
+            // memory, which frees the history values' registers early
+            if (!GROUPED) release_stage(empty0 + 8u * stage, lane);
             if (full_tile && mine) {
                 void* out = member_out<K, CB16, U>(A, first + m, ev, raw);
                 if (A.precise) {
@@ -347,7 +349,7 @@ __global__ void __launch_bounds__(Shape<CB16, K, GROUPED, GATED>::threads, Shape
                                                          acc, gate);
                 }
             }
-            if (!hold) release_stage(empty0 + 8u * stage, lane);
+            if (GROUPED && !hold) release_stage(empty0 + 8u * stage, lane);
         }
         if (GROUPED && hold) {
             const uint32_t last = stage_of(nb - 1);
