@@ -33,6 +33,15 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "extrapolation GB/s & % of HBM peak; µs per skipped step (all blocks), 1 GB300"
+# configurations timed after the headline (FLUX.1-dev 1024^2), each on its own
+# filled history: (preset, [(variant, hidden states fused)])
+OTHER_WORKLOADS = [
+    ("pixart", [("prediction-only", False), ("fused", True)]),
+    ("dit512", [("prediction-only", False)]),
+    ("dit256", [("fused", True), ("prediction-only", False)]),
+    ("dit256-k3", [("fused", True), ("prediction-only", False)]),
+    ("flux", [("fused", True)]),
+]
 NOMINAL_HBM_GBS = 7900.0
 KERNEL_SOURCES = ["paper_2608_23429_gb300/csrc/extrapolate_bulk.cu", "paper_2608_23429_gb300/csrc/bulk_kernel.cuh",
                   "paper_2608_23429_gb300/csrc/extrapolate.cu", "paper_2608_23429_gb300/csrc/direct_kernel.cuh",
@@ -153,10 +162,20 @@ def workload_description(w) -> dict:
                          if w.explicit_nodes else f"T={w.T}, full every r={w.r}")}
 
 
-def pick_window(w, orc):
-    """Walk the schedule to the first window of K equispaced nodes past the
+def full_mask(w, cb):
+    """The schedule's full steps (Sec. 3.3 set F plus warm-up), from the library."""
+    mask, _ = cb.cb_schedule_full(w.T, w.r, w.s0, w.s1, w.K)
+    return mask
+
+
+def pick_window(w, cb):
+    """The product's timed window: see window_of."""
+    return window_of(w, full_mask(w, cb))
+
+
+def window_of(w, mask):
+    """Walk a schedule mask to the first window of K equispaced nodes past the
     warm-up; return (full steps pushed in order, skipped steps that follow)."""
-    mask = orc.full_schedule(w.T, w.r, w.s0, w.s1, w.K)
     full = [s for s in range(w.T) if mask[s]]
     for k in range(w.K - 1, len(full) - 1):
         win = full[k - w.K + 1:k + 1]
@@ -182,6 +201,20 @@ def cpu_oracle_run(w, feats_host, wts, seconds: float, nthreads: int):
     return gbs, n, reps, el
 
 
+def oracle_parity(orc, host, wts, gpu_bits) -> dict:
+    """The oracle's fp64 prediction for the sampled elements (the first
+    gpu_bits.size of the CPU baseline's sample), rounded once to bf16, against
+    the GPU's bits."""
+    import numpy as np
+    n = gpu_bits.size
+    F = [h[:n] for h in host]
+    o64, _ = orc.extrapolate([F], wts, orc.BF16, orc.FP64, nthreads=os.cpu_count() or 1)
+    ref = orc.convert(o64[0], orc.FP64, orc.BF16)
+    Fd = np.array([(f.astype(np.uint32) << 16).view(np.float32).astype(np.float64) for f in F])
+    bound = (np.abs(np.asarray(wts, dtype=np.float64))[:, None] * np.abs(Fd)).sum(0)
+    return parity_stats(gpu_bits, ref, o64[0], bound)
+
+
 def cpu_model() -> str:
     """The host CPU's model name (lscpu, else /proc/cpuinfo)."""
     try:
@@ -203,8 +236,7 @@ def cpu_model() -> str:
 def sample_host_features(w, torch, wl, orc, n_elems: int, device):
     """A bounded contiguous sample of the largest tensor at K nodes (generator bytes)."""
     i = max(range(len(w.tensors)), key=lambda k: w.tensors[k].numel)
-    _, targets = pick_window(w, orc)
-    full, _ = pick_window(w, orc)
+    full, targets = window_of(w, orc.full_schedule(w.T, w.r, w.s0, w.s1, w.K))  # the oracle's own schedule
     nodes = full[-w.K:]
     host = []
     for s in nodes:
@@ -213,6 +245,95 @@ def sample_host_features(w, torch, wl, orc, n_elems: int, device):
     t_nodes = [w.timesteps[s] for s in nodes]
     wts = orc.weights(t_nodes, w.timesteps[targets[0]], w.t_min, w.t_max)
     return host, wts, i
+
+
+def parity_stats(gpu_bits, ref_bits, ref64, bound64) -> dict:
+    """bf16 results against the oracle: ulp distance of the bit patterns, with
+    exact cancellations (|gpu - exact| <= 2^-40 sum_j |w_j F_j|) counted apart."""
+    import numpy as np
+
+    def ordered(b):
+        b = b.astype(np.int64)
+        return np.where(b & 0x8000, -(b & 0x7FFF), b)
+
+    d = np.abs(ordered(gpu_bits) - ordered(ref_bits))
+    g64 = (gpu_bits.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    floor = np.abs(g64 - ref64) <= 2.0 ** -40 * bound64
+    return {"n": int(d.size), "exact": int((d == 0).sum()), "one_ulp": int((d == 1).sum()),
+            "floor": int(((d > 1) & floor).sum()), "bad": int(((d > 1) & ~floor).sum()),
+            "max_ulp": int(d.max()) if d.size else 0}
+
+
+def fill_window(torch, cb, wl, w, plan, cdt, pushed, dev, stream):
+    """The schedule's full steps up to the timed window, pushed in order."""
+    for s in pushed:
+        feats = [wl.trajectory(w, i, w.timesteps[s], s, dev) for i in range(len(w.tensors))]
+        torch.cuda.synchronize()
+        cb.cb_cache_push(plan, feats, cdt, w.timesteps[s], stream=stream)
+        stream.synchronize()
+        del feats
+
+
+def time_workload(torch, cb, wl, dev, name: str, variants, steps: int, warmup: int, peak: float) -> list:
+    """Skipped steps of one more workload in the launch configuration of the
+    headline: the same window walk, one launch per step, per-launch events on
+    the launching stream. variants: (label, fused) pairs on one filled history."""
+    w = wl.PRESETS[name]()
+    K = w.K
+    pushed, targets = pick_window(w, cb)
+    node_t = [w.timesteps[s] for s in full_mask(w, cb).nonzero()[0]]
+    cdt = cb.CB_BF16 if w.cache_dtype == "bf16" else cb.CB_FP32
+    tdt = torch.bfloat16 if w.cache_dtype == "bf16" else torch.float32
+    plan = cb.cb_plan_create(node_t, K, [(t.layer, t.branch, t.numel, t.group) for t in w.tensors], cdt,
+                             w.t_min, w.t_max)
+    cache = torch.empty(cb.cb_plan_cache_bytes(plan), dtype=torch.uint8, device=dev)
+    cb.cb_plan_bind_cache(plan, cache, cache.numel())
+    stream = torch.cuda.Stream(device=dev)
+    fill_window(torch, cb, wl, w, plan, cdt, pushed, dev, stream)
+    outs = [torch.empty(t.shape, dtype=tdt, device=dev) for t in w.tensors]
+    n_groups = cb.cb_plan_num_groups(plan)
+    slot_elems = sum(t.numel for t in w.tensors)
+    esz = 2 if w.cache_dtype == "bf16" else 4
+    t_targets = [w.timesteps[s] for s in targets]
+    rows = []
+    for label, fused in variants:
+        resid = [wl.hidden_state(w, g, dev) for g in range(n_groups)] if fused else None
+        resid_elems = sum(w.group_numel(g) for g in range(n_groups)) if fused else 0
+        bytes_step = slot_elems * esz * (K + 1) + resid_elems * 2 * 2
+        outs_p = cb.ptr_array(outs)
+        resid_p = cb.ptr_array(resid) if resid is not None else None
+        w0, w1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        w0.record(stream)
+        for k in range(warmup):
+            cb.cb_extrapolate(plan, t_targets[k % len(t_targets)], outs_p, cdt, resid_p, cb.CB_BF16, stream=stream)
+        w1.record(stream)
+        stream.synchronize()
+        # at least ~0.3 s of timed steps, so that the clock sampler sees the load
+        n = max(steps, int(0.3e3 / max(w0.elapsed_time(w1) / warmup, 1e-3)))
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+        with Clocks(torch.cuda.current_device()) as clk:
+            for k in range(n):
+                ev[k][0].record(stream)
+                cb.cb_extrapolate(plan, t_targets[k % len(t_targets)], outs_p, cdt, resid_p, cb.CB_BF16,
+                                  stream=stream)
+                ev[k][1].record(stream)
+            stream.synchronize()
+        clocks = clk.summary()
+        if cb.cb_plan_device_status(plan, stream=stream) != 0:
+            raise RuntimeError(f"device status set while timing {name}")
+        us = sorted(a.elapsed_time(b) * 1e3 for a, b in ev)
+        mean_us = sum(us) / len(us)
+        rows.append({"workload": w.name, "variant": label, "K": K, "fused_residual": bool(fused),
+                     "bytes_per_step": bytes_step, "us_per_step": round(mean_us, 2),
+                     "us_per_step_median": round(us[len(us) // 2], 2),
+                     "gbs": round(bytes_step / (mean_us * 1e-6) / 1e9, 2),
+                     "frac": round(bytes_step / (mean_us * 1e-6) / 1e9 / peak, 4), "steps": n,
+                     "clocks": {"sm_mhz": clocks["sm_mhz"], "reasons": clocks["reasons"]}})
+        del resid
+    cb.cb_plan_destroy(plan)
+    del cache, outs
+    torch.cuda.empty_cache()
+    return rows
 
 
 def run_reference(args):
@@ -287,8 +408,8 @@ def run_ours(args):
         targets = list(range(len(pushed), len(w.timesteps)))
         node_t = list(w.explicit_nodes)
     else:
-        pushed, targets = pick_window(w, orc)
-        node_t = [w.timesteps[s] for s in orc.full_schedule(w.T, w.r, w.s0, w.s1, K).nonzero()[0]]
+        pushed, targets = pick_window(w, cb)
+        node_t = [w.timesteps[s] for s in full_mask(w, cb).nonzero()[0]]
     tensors = [(t.layer, t.branch, t.numel, t.group) for t in w.tensors]
     cdt = cb.CB_BF16 if w.cache_dtype == "bf16" else cb.CB_FP32
     tdt = torch.bfloat16 if w.cache_dtype == "bf16" else torch.float32
@@ -298,12 +419,7 @@ def run_ours(args):
     cb.cb_plan_set_option(plan, cb.CB_OPT_KERNEL, {"auto": cb.CB_KERNEL_AUTO, "direct": cb.CB_KERNEL_DIRECT,
                                                    "bulk": cb.CB_KERNEL_BULK}[args.kernel])
     stream = torch.cuda.Stream(device=dev)
-    for s in pushed:  # full steps of the schedule up to the timed window
-        feats = [wl.trajectory(w, i, w.timesteps[s], s, dev) for i in range(len(w.tensors))]
-        torch.cuda.synchronize()
-        cb.cb_cache_push(plan, feats, cdt, w.timesteps[s], stream=stream)
-        stream.synchronize()
-        del feats
+    fill_window(torch, cb, wl, w, plan, cdt, pushed, dev, stream)  # full steps up to the timed window
     outs = [torch.empty(t.shape, dtype=tdt, device=dev) for t in w.tensors]
     slot_elems = sum(t.numel for t in w.tensors)
     esz = 2 if w.cache_dtype == "bf16" else 4
@@ -428,10 +544,20 @@ def run_ours(args):
     peak, peak_src = measured_peaks()
     achieved = bytes_step / (avg_kern / 1e3) / 1e9
 
+    # ---- the timed step once more at the first target: its predictions for the
+    # largest tensor (the CPU baseline's sample) are checked against the oracle
+    check = None
+    if rank == 0 and ws == 1 and not args.no_cpu and args.step == "skip" and not tiny:
+        ti = max(range(len(w.tensors)), key=lambda k: w.tensors[k].numel)
+        extrapolate_at(t_targets[0])
+        stream.synchronize()
+        n_chk = min(args.cpu_elems, w.tensors[ti].numel)
+        check = (ti, outs[ti].reshape(-1)[:n_chk].cpu().view(torch.int16).numpy().view("uint16").copy())
+
     # ---- the whole online loop of Alg. 1 over the schedule, ring evolving
     sched = None
     if args.step == "skip" and args.schedule_reps > 0 and not tiny:
-        sched = run_schedule_loop(args, torch, cb, wl, orc, w, plan, cdt, dev, stream, extrapolate_at, bytes_step)
+        sched = run_schedule_loop(args, torch, cb, wl, w, plan, cdt, dev, stream, extrapolate_at, bytes_step)
 
     # ---- end to end through the public API with host buffers: upload the K
     # cached feature sets from pinned host memory (push), extrapolate, read the
@@ -441,8 +567,13 @@ def run_ours(args):
         e2e = run_e2e(args, torch, cb, wl, w, plan, cdt, tdt, dev, pushed, t_targets, bytes_step, ws, fused)
 
     cpu = None
-    if rank == 0 and ws == 1 and not args.no_cpu and args.step == "skip" and not tiny:
+    parity = None
+    if check is not None:
         host, wts, ti = sample_host_features(w, torch, wl, orc, args.cpu_elems, dev)
+        assert ti == check[0]
+        parity = oracle_parity(orc, host, wts, check[1])
+        parity["sample"] = (f"{check[1].size} elements of tensor {ti} ({w.tensors[ti].shape}) at the first timed "
+                            f"target, predicted by one more launch after the timed steps")
         threads = os.cpu_count() or 1
         gbs, n, reps, el = cpu_oracle_run(w, host, wts, args.cpu_seconds, threads)
         gbs1, _, reps1, el1 = cpu_oracle_run(w, host, wts, args.cpu_seconds / 2, 1)
@@ -453,6 +584,18 @@ def run_ours(args):
                          f"on 1 thread (fp64 oracle, bf16 in/out)"}
 
     cb.cb_plan_destroy(plan)
+    del outs, resid, cache
+    torch.cuda.empty_cache()
+
+    # ---- the other configurations' skipped steps (same launch configuration)
+    others = None
+    if (rank == 0 and ws == 1 and args.step == "skip" and args.config == "flux" and args.scale == 1
+            and not args.gated and args.launch == "per-step" and args.kernel == "auto" and args.workload_steps > 0):
+        peak_now, _ = measured_peaks()
+        others = []
+        for name, variants in OTHER_WORKLOADS:
+            others += time_workload(torch, cb, wl, dev, name, variants, args.workload_steps, 3, peak_now)
+
     if rank == 0:
         desc = workload_description(w)
         desc.update({"bytes_per_step": bytes_step, "fused_residual": fused, "step": args.step,
@@ -478,7 +621,7 @@ def run_ours(args):
                                      and not args.gated else None),
                          "kernel": kernel_name,
                          "avg_launch_us": round(avg_kern * 1e3, 2)},
-            "schedule_loop": sched,
+            "schedule_loop": sched, "parity": parity, "workloads": others,
             "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks, "gpu_launches": args.steps * launches_per_step,
         }
         print(json.dumps(line))
@@ -499,13 +642,13 @@ def host_memory_is_device_mapped(ptr: int) -> bool:
     return rc == 0 and dptr.value == ptr
 
 
-def run_schedule_loop(args, torch, cb, wl, orc, w, plan, cdt, dev, stream, extrapolate_at, bytes_step):
+def run_schedule_loop(args, torch, cb, wl, w, plan, cdt, dev, stream, extrapolate_at, bytes_step):
     """Alg. 1's online stage over the whole schedule, `schedule_reps` times from an
     empty history: warm-up and full steps push that step's features (generated
     once, before the timed loops), skipped steps extrapolate with the ring as it
     evolves. Each launch is bracketed by events on the launching stream; only
     the skipped steps count toward the metric, the pushes are timed apart."""
-    mask = orc.full_schedule(w.T, w.r, w.s0, w.s1, w.K)
+    mask = full_mask(w, cb)
     full = [s for s in range(w.T) if mask[s]]
     skipped = [s for s in range(w.T) if not mask[s]]
     feats = {}
@@ -666,6 +809,8 @@ def main():
     ap.add_argument("--schedule-reps", type=int, default=5,
                     help="repetitions of the whole schedule loop (0: skip it)")
     ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--workload-steps", type=int, default=20,
+                    help="timed steps of each other configuration after the headline (0: skip them)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     args = ap.parse_args()
