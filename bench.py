@@ -400,6 +400,8 @@ def run_ours(args):
     w = wl.PRESETS[args.config]()
     if args.scale > 1:
         w = wl.scaled(w, args.scale)
+    if args.history:
+        w.K = args.history
     K = w.K
     tiny = bool(w.explicit_nodes)
     if tiny:  # explicit nodes and targets instead of a schedule; L2-resident, a latency case
@@ -590,7 +592,8 @@ def run_ours(args):
     # ---- the other configurations' skipped steps (same launch configuration)
     others = None
     if (rank == 0 and ws == 1 and args.step == "skip" and args.config == "flux" and args.scale == 1
-            and not args.gated and args.launch == "per-step" and args.kernel == "auto" and args.workload_steps > 0):
+            and not args.history and not args.gated and args.launch == "per-step" and args.kernel == "auto"
+            and args.workload_steps > 0):
         peak_now, _ = measured_peaks()
         others = []
         for name, variants in OTHER_WORKLOADS:
@@ -800,6 +803,8 @@ def main():
                     help="type of the full step's features (--step full / full-fused)")
     ap.add_argument("--kernel", default="auto", choices=["auto", "direct", "bulk"],
                     help="skipped-step kernel variant (both compute identical bits)")
+    ap.add_argument("--history", type=int, default=0,
+                    help="history size K instead of the workload's own (1..8; changes the schedule's warm-up)")
     ap.add_argument("--scale", type=int, default=1,
                     help="divide every tensor's token count (small cases for profiling only)")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)

@@ -244,11 +244,6 @@ __device__ __forceinline__ void store_f32x8(void* p, long long e, const float (&
     q[1] = make_uint4(__float_as_uint(v[4]), __float_as_uint(v[5]), __float_as_uint(v[6]), __float_as_uint(v[7]));
 }
 
-__device__ __forceinline__ void set_half(uint32_t (&pk)[4], int e, uint16_t h) {
-    uint32_t& w = pk[e >> 1];
-    w = (e & 1) ? ((w & 0x0000FFFFu) | ((uint32_t)h << 16)) : ((w & 0xFFFF0000u) | h);
-}
-
 // Running sums of one item across its members (the fused hidden-state update):
 // fast path x = sum_b s_b, y = sum_b a_b; compensated path x + y is the
 // unevaluated sum (running value and its error).
@@ -384,7 +379,11 @@ __device__ __forceinline__ void member_fast(const ExtrapArgs& A, long long moff,
             unsigned bad = 0;
 #pragma unroll
             for (int e = 0; e < 8; ++e) bad |= guard_ok(a[e], s[e]) ? 0u : (1u << e);
-            while (bad) {  // rare: recompute the failing elements with Dot2
+            store_bf16x8(out, ev[u], pk);
+            // rare: the failing elements get their Dot2 value, stored by this
+            // thread over the fast-path bf16 it has just written (the vector is
+            // dead by then, so the loop keeps nothing of the fast path live)
+            while (bad) {
                 const int e = __ffs(bad) - 1;
                 bad &= bad - 1;
                 float hi, lo;
@@ -394,9 +393,8 @@ __device__ __forceinline__ void member_fast(const ExtrapArgs& A, long long moff,
                     exact_from_raw<K, CB16, UV>(A, raw, u, e, hi, lo);
                 else
                     exact_member<CB16>(A, K, moff, ev[u] + e, hi, lo);
-                set_half(pk, e, bf16_of_pair(hi, lo));
+                reinterpret_cast<uint16_t*>(out)[ev[u] + e] = bf16_of_pair(hi, lo);
             }
-            store_bf16x8(out, ev[u], pk);
         }
         if (accumulate) {
             float g[8];
@@ -447,6 +445,8 @@ __device__ __forceinline__ void resid_fast(const ExtrapArgs& A, int it, const lo
         if (!pass)
 #pragma unroll
             for (int e = 0; e < 8; ++e) bad |= guard_ok(b[e], t[e]) ? 0u : (1u << e);
+        store_bf16x8(resid, ev[u], pk);
+        // rare: Dot2 values stored over the fast-path bf16 just written
         while (bad) {
             const int e = __ffs(bad) - 1;
             bad &= bad - 1;
@@ -455,9 +455,8 @@ __device__ __forceinline__ void resid_fast(const ExtrapArgs& A, int it, const lo
             for (int i = 1; i < 8; ++i) xe = (e == i) ? x[i] : xe;
             float hi, lo;
             exact(u, e, xe, hi, lo);
-            set_half(pk, e, bf16_of_pair(hi, lo));
+            reinterpret_cast<uint16_t*>(resid)[ev[u] + e] = bf16_of_pair(hi, lo);
         }
-        store_bf16x8(resid, ev[u], pk);
     }
 }
 
