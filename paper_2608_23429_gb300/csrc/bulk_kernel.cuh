@@ -146,9 +146,13 @@ __device__ __forceinline__ void release_stage(uint32_t empty_bar, int lane) {
 // holding, hidden-state staging); prediction-only launches compile without
 // that bookkeeping. GATED (with GROUPED): the hidden state receives g_b * P_b,
 // with a per-(batch, channel) gate per member.
-template <int K, bool CB16, bool GROUPED, bool GATED>
+// ONE: the full-step epilogue (copy_out with bf16 hidden states or none): a
+// one-entry history of weight 1, whose member step needs no weighted sum
+// (member_one); compiled apart so that each kernel carries only its own path.
+template <int K, bool CB16, bool GROUPED, bool GATED, bool ONE = false>
 __global__ void __launch_bounds__(Shape<CB16, K, GROUPED, GATED>::threads, Shape<CB16, K, GROUPED, GATED>::ctas_per_sm)
     extrapolate_bulk_kernel(const __grid_constant__ ExtrapArgs A) {
+    static_assert(!ONE || K == 1, "the epilogue is a one-entry history");
     extern __shared__ __align__(128) unsigned char smem[];
     constexpr int NCW = Shape<CB16, K, GROUPED, GATED>::consumer_warps;
     constexpr int NCT = Shape<CB16, K, GROUPED, GATED>::consumers;
@@ -327,7 +331,9 @@ __global__ void __launch_bounds__(Shape<CB16, K, GROUPED, GATED>::threads, Shape
             if (!GROUPED) release_stage(empty0 + 8u * stage, lane);
             if (full_tile && mine) {
                 void* out = member_out<K, CB16, U>(A, first + m, ev, raw);
-                if (A.precise) {
+                if constexpr (ONE) {
+                    if (resid != nullptr) member_one<K, CB16, U, GATED>(raw, acc, gate);
+                } else if (A.precise) {
                     member_precise<K, CB16, U, GATED>(A, out, ev, raw, resid != nullptr, acc, gate);
                 } else if constexpr (GROUPED) {
                     auto exact = [&](int v, int e, float& hi, float& lo) {
@@ -360,7 +366,7 @@ __global__ void __launch_bounds__(Shape<CB16, K, GROUPED, GATED>::threads, Shape
                     load_x8(resid, A.resid_bf16, ev[v], x);
             };
             if (!mine) {
-            } else if (A.precise) {
+            } else if (!ONE && A.precise) {
                 resid_precise<U>(A, ev, acc, resid, xload);
             } else {
                 // Dot2 of x + sum_b P_b for one element, from the held stages
@@ -391,7 +397,7 @@ __global__ void __launch_bounds__(Shape<CB16, K, GROUPED, GATED>::threads, Shape
                     }
                     two_sum(tp, tc, hi, lo);
                 };
-                resid_fast<K, U>(A, it, ev, acc, resid, xload, exact);
+                resid_fast<K, U>(A, it, ev, acc, resid, xload, exact, ONE ? A.w_guard[0] : 1.0f);
             }
             fence_generic_to_async();
             __syncwarp();

@@ -413,17 +413,50 @@ __device__ __forceinline__ void member_fast(const ExtrapArgs& A, long long moff,
     }
 }
 
+// Full-step epilogue (a one-entry history of weight 1): member features f,
+// taken exactly, added into the hidden-state sums, acc.x += g f and the
+// unscaled bound acc.y += |g f| (g = 1 without gates). resid_fast scales the
+// bound with yscale = w_guard[0] = 3 u (1.01) 2^9, the scaled bound the general
+// path would have accumulated for K = 1.
+template <int K, bool CB16, int UV, bool GATED = false, typename Gate = NoGate>
+__device__ __forceinline__ void member_one(const RawVecs<K, CB16, UV>& raw, Acc<UV>& acc, Gate gate = {}) {
+    static_assert(K == 1, "a one-entry history");
+#pragma unroll
+    for (int u = 0; u < UV; ++u) {
+        float g[8];
+        if constexpr (GATED) gate(u, g);  // first: each feature is then unpacked as it is used
+        const uint32_t w[8] = {raw[u][0][0].x, raw[u][0][0].y, raw[u][0][0].z, raw[u][0][0].w,
+                               raw[u][0][CB16 ? 0 : 1].x, raw[u][0][CB16 ? 0 : 1].y, raw[u][0][CB16 ? 0 : 1].z,
+                               raw[u][0][CB16 ? 0 : 1].w};
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const float f = CB16 ? __uint_as_float((e & 1) ? (w[e >> 1] & 0xFFFF0000u) : (w[e >> 1] << 16))
+                                 : __uint_as_float(w[e]);
+            if constexpr (GATED) {
+                acc.x[u][e] = fmaf(g[e], f, acc.x[u][e]);
+                acc.y[u][e] = fmaf(fabsf(g[e]), fabsf(f), acc.y[u][e]);
+            } else {
+                acc.x[u][e] += f;
+                acc.y[u][e] += fabsf(f);
+            }
+        }
+    }
+}
+
 // Fast path: hidden state <- bf16(x + sum_b s_b), guarded like the members.
 // xload(u, x) supplies the 8 hidden-state values of vector u (global or shared
 // memory); exact(u, e, x_e, hi, lo) recomputes one guarded element with Dot2.
+// yscale: factor that turns acc.y into the scaled bound (1 when the members
+// accumulated scaled bounds; w_guard[0] after member_one's unscaled sums).
 template <int K, int UV, typename XLoad, typename Exact>
 __device__ __forceinline__ void resid_fast(const ExtrapArgs& A, int it, const long long (&ev)[UV],
-                                           const Acc<UV>& acc, void* resid, XLoad xload, Exact exact) {
+                                           const Acc<UV>& acc, void* resid, XLoad xload, Exact exact,
+                                           float yscale = 1.0f) {
     // the test g_res (sum_b a_b + |x|) <= 2^-9 |t|, g_res = (K + nb + 3) u 1.01,
     // on the scaled bounds acc.y = (K+2) u 1.01 2^9 sum_b a_b:
     // q acc.y + r |x| <= |t| with q = (K + nb + 3) / (K + 2), r = g_res 2^9
     const float kn = (float)(K + A.nb[it] + 3);
-    const float q = kn * (1.0f / (float)(K + 2)) * 1.0000005f;  // rounded up past fp32 error
+    const float q = kn * (1.0f / (float)(K + 2)) * 1.0000005f * yscale;  // rounded up past fp32 error
     const float r = kn * (kU * 1.01f * 512.0f);
 #pragma unroll
     for (int u = 0; u < UV; ++u) {

@@ -72,7 +72,27 @@ __device__ __forceinline__ void item_vectors(const ExtrapArgs& A, int it, const 
             RawVecs<K, CB16, UV> raw;
             load_member<K, CB16, UV>(A, A.m_off[first + m], ev, raw);
             void* out = member_out<K, CB16, UV>(A, first + m, ev, raw);
-            if constexpr (GATED) {
+            // full-step epilogue from bf16 features: exact features, no weighted
+            // sum (the bulk kernel's ONE path; from fp32 features both kernels
+            // take the general path)
+            bool one = false;
+            if constexpr (K == 1 && CB16) {
+                one = A.copy_out != 0;
+                if (one && resid) {
+                    if constexpr (GATED) {
+                        float g[UV][8];
+                        load_gates<UV>(A, first + m, gi, g);
+                        member_one<K, CB16, UV, true>(raw, acc, [&](int u, float (&gv)[8]) {
+#pragma unroll
+                            for (int e = 0; e < 8; ++e) gv[e] = g[u][e];
+                        });
+                    } else {
+                        member_one<K, CB16, UV>(raw, acc);
+                    }
+                }
+            }
+            if (one) {
+            } else if constexpr (GATED) {
                 float g[UV][8];
                 load_gates<UV>(A, first + m, gi, g);
                 member_fast<K, CB16, UV, false, true>(A, A.m_off[first + m], out, ev, raw,
@@ -90,7 +110,8 @@ __device__ __forceinline__ void item_vectors(const ExtrapArgs& A, int it, const 
                 A, it, ev, acc, resid, [&](int u, float (&x)[8]) { load_x8(resid, true, ev[u], x); },
                 [&](int u, int e, float xe, float& hi, float& lo) {
                     exact_resid<CB16>(A, K, it, ev[u] + e, xe, hi, lo);
-                });
+                },
+                (K == 1 && A.copy_out) ? A.w_guard[0] : 1.0f);
     }
 }
 

@@ -5,16 +5,30 @@
 namespace cbk {
 namespace {
 
+// The full-step epilogue from bf16 features (a copy_out launch without
+// compensated hidden states) runs the ONE instantiation; from fp32 features
+// the general path (see extrapolate_bulk.cu).
 template <int K, bool CB16>
 cudaError_t launch_gk(const ExtrapArgs& a, int grid, size_t smem, cudaStream_t s) {
+    if constexpr (K == 1 && CB16) {
+        if (a.copy_out && !a.precise) {
+            extrapolate_bulk_kernel<K, CB16, true, true, true><<<grid, Shape<CB16, K, true, true>::threads, smem, s>>>(a);
+            return cudaGetLastError();
+        }
+    }
     extrapolate_bulk_kernel<K, CB16, true, true><<<grid, Shape<CB16, K, true, true>::threads, smem, s>>>(a);
     return cudaGetLastError();
 }
 
 template <int K, bool CB16>
 cudaError_t prepare_gk(size_t smem) {
-    return cudaFuncSetAttribute(extrapolate_bulk_kernel<K, CB16, true, true>,
-                                cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = cudaFuncSetAttribute(extrapolate_bulk_kernel<K, CB16, true, true>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if constexpr (K == 1 && CB16)
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(extrapolate_bulk_kernel<K, CB16, true, true, true>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    return e;
 }
 
 #define CB_K_SWITCH(K, CALL)                  \

@@ -532,25 +532,28 @@ def test_direct_and_bulk_kernels_bit_identical(cb, H, name):
     torch.cuda.empty_cache()
 
 
-def test_bulk_wait_limit_reports_and_recovers(cb, H):
+@pytest.mark.parametrize("K,fused", [(4, False), (2, False), (3, True)])
+def test_bulk_wait_limit_reports_and_recovers(cb, H, K, fused):
     """The failure path of the bulk kernel's bounded waits, without a fault: the
     producer announces every CTA's first unit but never issues its copies (a
     flag that nothing sets), so the consumers' wait runs out after the limit.
     The kernel must record it in the status word and return; the context stays
-    usable and the next launch is correct and clean."""
+    usable and the next launch is correct and clean. Shapes: predictions only
+    with one CTA per SM (K = 4) and with two (K = 2), hidden states fused with
+    two CTAs per SM (K = 3)."""
     import time
     w = workloads.scaled(workloads.pixart(), 16)
-    walk = H.Walk(w, kernel="bulk")
-    mask, skipped = H.schedule_steps(w, w.K)
-    for s in range(skipped[0]):
-        if mask[s]:
-            walk.push(w.timesteps[s], s)
-    t = w.timesteps[skipped[0]]
+    nodes = [999.0 - 45.0 * k for k in range(K)]
+    walk = H.Walk(w, K=K, node_t=nodes, kernel="bulk")
+    for k, t in enumerate(nodes):
+        walk.push(t, k)
+    t = nodes[-1] - 30.0
     outs = [torch.empty(s.shape, dtype=torch.bfloat16, device="cuda") for s in w.tensors]
+    resid = [workloads.hidden_state(w, g, "cuda") for g in range(walk.n_groups)] if fused else None
     cb.cb_plan_set_option(walk.plan, cb.CB_OPT_WAIT_NS, 20_000_000)  # 20 ms
     cb.cb_plan_set_option(walk.plan, cb.CB_OPT_TEST_WITHHOLD, 1)
     t0 = time.perf_counter()
-    cb.cb_extrapolate(walk.plan, t, outs, cb.CB_BF16)
+    cb.cb_extrapolate(walk.plan, t, outs, cb.CB_BF16, resid, cb.CB_BF16)
     torch.cuda.synchronize()
     elapsed = time.perf_counter() - t0
     st = cb.cb_plan_device_status(walk.plan)
@@ -560,8 +563,11 @@ def test_bulk_wait_limit_reports_and_recovers(cb, H):
     assert cb.cb_plan_device_status(walk.plan) == 0  # the read cleared it
     cb.cb_plan_set_option(walk.plan, cb.CB_OPT_TEST_WITHHOLD, 0)
     cb.cb_plan_set_option(walk.plan, cb.CB_OPT_WAIT_NS, 10 ** 9)
-    outs, _, _ = walk.extrapolate(t)
-    _assert_ok(walk.expected_and_compare(t, outs, None, None)[0], "after timeout")
+    outs, resid, rh = walk.extrapolate(t, fused=fused, salt=K)
+    so, sr, _ = walk.expected_and_compare(t, outs, resid, rh)
+    _assert_ok(so, ("after timeout", K))
+    if fused:
+        _assert_ok(sr, ("after timeout, hidden states", K))
     walk.close()
 
 
