@@ -48,8 +48,8 @@ namespace {
 // Thread map. With one CTA per SM, one 8-element vector per consumer thread
 // and tile: 16 consumer warps for bf16 tiles (512 vectors; 17 warps cap
 // registers at 96), 8 for fp32 tiles (256 vectors). Launches that carry few
-// bytes per unit (K = 1, and bf16 launches with small K: bulk_ctas_per_sm) pay
-// the consumers' fixed cost per unit more often; they run two CTAs of 8
+// bytes per unit (most K = 1 launches, and bf16 launches with small K: see
+// bulk_ctas_per_sm) pay the consumers' fixed cost per unit more often; they run two CTAs of 8
 // consumer warps per SM (two independent pipelines), bf16 threads taking two
 // vectors per tile. An earlier map of 8 consumer warps with two vectors each
 // on one CTA left the launches with hidden states issue-bound.
