@@ -177,6 +177,8 @@ __global__ void __launch_bounds__(Shape<CB16, K, GROUPED, GATED>::threads, Shape
     }
     __syncthreads();
 
+    // the stage stays held through the member's arithmetic (see the consumers)
+    constexpr bool LATE = GROUPED || (CB16 && K >= 7);
     const int C = GROUPED ? A.stage_chunks : K;
     const uint32_t stage_bytes = (uint32_t)C * kChunkBytes + (GATED ? A.stage_gate_bytes : 0u);
     if (warp == NCW) {  // ---------------------------------- producer
@@ -326,16 +328,17 @@ __global__ void __launch_bounds__(Shape<CB16, K, GROUPED, GATED>::threads, Shape
             };
             // prediction-only launches release the stage as soon as it is read
             // and recompute guarded elements from registers; grouped launches
-            // keep the stage until the member is done and recompute from shared
-            // memory, which frees the history values' registers early
-            if (!GROUPED) release_stage(empty0 + 8u * stage, lane);
+            // and bf16 ones with K >= 7 keep the stage until the member is done
+            // and recompute from shared memory, which frees the history values'
+            // registers early (bf16 K >= 7 would otherwise spill under the cap)
+            if (!LATE) release_stage(empty0 + 8u * stage, lane);
             if (full_tile && mine) {
                 void* out = member_out<K, CB16, U>(A, first + m, ev, raw);
                 if constexpr (ONE) {
                     if (resid != nullptr) member_one<K, CB16, U, GATED>(raw, acc, gate);
                 } else if (A.precise) {
                     member_precise<K, CB16, U, GATED>(A, out, ev, raw, resid != nullptr, acc, gate);
-                } else if constexpr (GROUPED) {
+                } else if constexpr (LATE) {
                     auto exact = [&](int v, int e, float& hi, float& lo) {
                         const size_t off = (size_t)(ev[v] - e0 + e) * ES;
                         float p = 0.0f, cc = 0.0f;
@@ -355,7 +358,7 @@ __global__ void __launch_bounds__(Shape<CB16, K, GROUPED, GATED>::threads, Shape
                                                          acc, gate);
                 }
             }
-            if (GROUPED && !hold) release_stage(empty0 + 8u * stage, lane);
+            if (LATE && !hold) release_stage(empty0 + 8u * stage, lane);
         }
         if (GROUPED && hold) {
             const uint32_t last = stage_of(nb - 1);
