@@ -45,7 +45,8 @@ OTHER_WORKLOADS = [
 NOMINAL_HBM_GBS = 7900.0
 KERNEL_SOURCES = ["paper_2608_23429_gb300/csrc/extrapolate_bulk.cu", "paper_2608_23429_gb300/csrc/bulk_kernel.cuh",
                   "paper_2608_23429_gb300/csrc/extrapolate.cu", "paper_2608_23429_gb300/csrc/direct_kernel.cuh",
-                  "paper_2608_23429_gb300/csrc/cb_math.cuh", "paper_2608_23429_gb300/csrc/cb_device.h"]
+                  "paper_2608_23429_gb300/csrc/cb_math.cuh", "paper_2608_23429_gb300/csrc/cb_device.h",
+                  "paper_2608_23429_gb300/csrc/cb_async.cuh"]
 
 
 def kernel_hash() -> str:
@@ -707,6 +708,10 @@ def run_e2e(args, torch, cb, wl, w, plan, cdt, tdt, dev, pushed, t_targets, byte
     host_resid = [wl.hidden_state(w, g, dev).cpu().pin_memory() for g in range(n_groups)] if fused else None
     mode = args.e2e_mode
     if mode == "zerocopy" and not host_memory_is_device_mapped(host_outs[0].data_ptr()):
+        mode = "copy"
+    # hidden states are read by the bulk kernel's bulk copies, which this
+    # bench only drives from device memory: fused steps stage them instead
+    if fused:
         mode = "copy"
     stream = torch.cuda.Stream(device=dev)
     slot = sum(t.numel for t in w.tensors) * (2 if w.cache_dtype == "bf16" else 4)

@@ -40,6 +40,7 @@
 // no fault and nothing in flight.
 #pragma once
 
+#include "cb_async.cuh"
 #include "cb_math.cuh"
 
 namespace cbk {
@@ -63,71 +64,6 @@ struct Shape {
 constexpr int kChunkBytes = 8192;   // one history entry's share of a tile
 constexpr int kBarrierBytes = 256;  // full[S] and empty[S] barriers, S <= kMaxStages
 static_assert(2 * 8 * kMaxStages <= kBarrierBytes, "barrier block holds every stage's barriers");
-constexpr unsigned long long kMinDrainNs = 10000000ull;  // copies land in microseconds
-constexpr unsigned long long kMaxWaitNs = 60000000000ull;  // no wait outlives a minute
-
-__device__ __forceinline__ uint32_t smem_addr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
-
-__device__ __forceinline__ unsigned long long now_ns() {
-    unsigned long long t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    return t;
-}
-
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(bar), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-
-// Wait for the phase with the given parity to complete, for at most limit_ns
-// (never more than kMaxWaitNs).
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, unsigned long long limit_ns) {
-    if (limit_ns > kMaxWaitNs) limit_ns = kMaxWaitNs;
-    if (mbar_try_wait(bar, parity)) return true;
-    const unsigned long long t0 = now_ns();
-    while (!mbar_try_wait(bar, parity))
-        if (now_ns() - t0 > limit_ns) return false;
-    return true;
-}
-
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
-}
-
-// Global -> shared bulk copy completing `bytes` transaction bytes on `bar`.
-// dst, src 16-byte aligned; bytes a multiple of 16.
-__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
-    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                     dst),
-                 "l"(src), "r"(bytes), "r"(bar)
-                 : "memory");
-}
-
-__device__ __forceinline__ void record(int* status, int code) {
-    if (status) atomicOr(status, code);
-}
-
-// Orders this thread's earlier generic-proxy accesses of shared memory before
-// later async-proxy accesses (the bulk copies that refill a released stage).
-__device__ __forceinline__ void fence_generic_to_async() {
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
-
 // A consumer warp hands one stage back to the producer: every lane fences its
 // shared-memory reads of the stage against the async proxy, then lane 0
 // arrives on the stage's empty barrier. The refill that follows is an
