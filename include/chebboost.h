@@ -185,6 +185,53 @@ int cb_extrapolate_ring(cb_plan* plan, const double* slot_t, int head, double t_
                         void* const* outs, cb_dtype out_dtype, void* const* resid,
                         cb_dtype resid_dtype, void* stream);
 
+/* The skipped step of cb_extrapolate_ring for callers that may not allocate
+ * device memory. The paper has no counterpart: this is a library convenience.
+ * Who needs it: an operator running inside a framework or inference engine
+ * that lays out every device buffer ahead of time. Such an operator is handed
+ * its input and output buffers and must not call cudaMalloc. The same holds
+ * for a process whose memory pool has already reserved the GPU. Such a caller
+ * can hold the history in a buffer of exactly K slots, but it cannot add the
+ * CB_STATUS_BYTES status block that cb_plan_bind_cache asks for. This call
+ * needs neither: the plan need not be bound, and the kernel records its
+ * device-side events in a block the library holds itself.
+ *
+ * plan: a plan from cb_plan_create. Only its tensor descriptors, K, time
+ *       interval, node table and options are used: its own history is
+ *       neither read nor changed.
+ * hist: device pointer to the caller's history buffer, CB_CACHE_ALIGN-aligned,
+ *       laid out like the arena's first K slots (slot p at p * slot_bytes,
+ *       slot_bytes = (cb_plan_cache_bytes(plan) - CB_STATUS_BYTES) / K).
+ *       hist_bytes: its size, at least K * slot_bytes.
+ * slot_t, head, t_target, outs, out_dtype, resid, resid_dtype, stream:
+ *       as cb_extrapolate_ring. Every slot must hold an entry.
+ * status: host pointer (may be NULL). It receives the launch's device status
+ *       word (CB_DEV_* codes, 0 = none) once the stream has reached the end
+ *       of this call. The value arrives by an asynchronous device-to-host
+ *       copy when *status is pinned memory. With ordinary memory the copy,
+ *       and thus this call, waits for the launch to finish.
+ *
+ * Allocation: the call allocates no device memory and no pinned host memory.
+ * Its status block is a file-scope device array of CB_STATUS_BYTES (256) bytes. Every GPU that
+ * loads the library holds it until the process exits. A call uses one 4-byte
+ * word of it whatever the workload's size, so no workload can outgrow it. The
+ * call still rejects a history buffer smaller than the K slots (CB_ERR_ARG),
+ * sizes beyond the CB_MAX_* limits and device ordinals from 64 up
+ * (CB_ERR_LIMIT).
+ * Set-up: the first call on each device looks up the block's device address
+ * there (cudaGetSymbolAddress, with that device current). Make that first call
+ * before any stream capture begins.
+ * Sharing: every call on a device uses the same word. Each launch clears it
+ * first on its own stream. Calls that overlap on the GPU (different streams,
+ * no ordering between them) race on it: one may clear or read another's
+ * code. Their outputs are unaffected.
+ * Errors: as cb_extrapolate_ring (CB_ERR_UNBOUND excepted), plus CB_ERR_ALIGN
+ * for hist and CB_ERR_CUDA when the status block cannot be reached. A
+ * CB_ERR_CUDA from the status read-back comes after the launch was enqueued. */
+int cb_extrapolate_noalloc(cb_plan* plan, const void* hist, size_t hist_bytes, const double* slot_t,
+                           int head, double t_target, void* const* outs, cb_dtype out_dtype,
+                           void* const* resid, cb_dtype resid_dtype, int* status, void* stream);
+
 /* Shapes of the branch tensors, needed by the gated calls: bth[3*i + 0..2] =
  * batch, tokens, hidden of tensor i (their product must be its numel;
  * tokens * hidden < 2^32). Tensors of one residual group must share tokens

@@ -48,6 +48,7 @@ _sig = {
     "cb_cache_push": ([_P, _PP, _I, _D, _P], _I),
     "cb_extrapolate": ([_P, _D, _PP, _I, _PP, _I, _P], _I),
     "cb_extrapolate_ring": ([_P, _P, _I, _D, _PP, _I, _PP, _I, _P], _I),
+    "cb_extrapolate_noalloc": ([_P, _P, _SZ, _P, _I, _D, _PP, _I, _PP, _I, _P, _P], _I),
     "cb_extrapolate_weights": ([_P, _P, _PP, _I, _PP, _I, _P], _I),
     "cb_plan_set_shapes": ([_P, _P], _I),
     "cb_extrapolate_gated": ([_P, _D, _PP, _I, _PP, _I, _PP, _I, _P], _I),
@@ -225,6 +226,24 @@ def cb_extrapolate_ring(plan, slot_t, head: int, t_target: float, outs, out_dtyp
     _check(_lib.cb_extrapolate_ring(plan, slot_t.ctypes.data, head, float(t_target),
                                     _ptrs(plan, outs, _TENSORS, c, "outs"), out_dtype,
                                     _ptrs(plan, resid, _GROUPS, c, "resid"), resid_dtype, _stream(stream)), c)
+
+
+def cb_extrapolate_noalloc(plan, hist, hist_bytes: int, slot_t, head: int, t_target: float, outs, out_dtype: int,
+                           resid=None, resid_dtype: int = CB_BF16, status=None, stream=None) -> None:
+    """The skipped step of cb_extrapolate_ring on a caller's history buffer
+    ``hist`` (the K slots, no status block; the plan need not be bound), for
+    callers that may not allocate device memory. ``status``: None, or a host
+    buffer (pinned keeps the call asynchronous) that receives the launch's
+    device status word once the stream gets there."""
+    c = "cb_extrapolate_noalloc"
+    slot_t = _f64(slot_t).ravel()
+    d = _dims(plan)
+    if d is not None and slot_t.size != d[_K]:  # the library reads K slot times
+        raise CbError(CB_ERR_ARG, f"{c} ({slot_t.size} slot times for K = {d[_K]})")
+    _check(_lib.cb_extrapolate_noalloc(plan, _addr(hist), int(hist_bytes), slot_t.ctypes.data, head,
+                                       float(t_target), _ptrs(plan, outs, _TENSORS, c, "outs"), out_dtype,
+                                       _ptrs(plan, resid, _GROUPS, c, "resid"), resid_dtype, _addr(status),
+                                       _stream(stream)), c)
 
 
 def cb_extrapolate_weights(plan, w_logical, outs, out_dtype: int, resid=None, resid_dtype: int = CB_BF16,

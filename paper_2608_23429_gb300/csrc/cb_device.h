@@ -114,4 +114,10 @@ cudaError_t launch_extrapolate_bulk_gated(const ExtrapArgs& a, int K, bool cache
 cudaError_t launch_push(const PushArgs& a, bool src_bf16, bool dst_bf16, int grid, cudaStream_t s);
 cudaError_t push_blocks_per_sm(bool src_bf16, bool dst_bf16, int* blocks);
 
+// Status word of cb_extrapolate_noalloc in the library's own device block
+// (static_status.cu): its device address on `device`, which must be the
+// current device. The first call per device looks the address up.
+constexpr int kMaxStatusDevices = 64;
+cudaError_t noalloc_status_word(int device, int** word);
+
 }  // namespace cbk

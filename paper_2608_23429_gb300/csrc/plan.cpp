@@ -284,16 +284,33 @@ int clear_status_once(cb_plan* p, void* stream) {
     return CB_OK;
 }
 
+// A history buffer given with the call instead of the bound arena, and the
+// status word its launch records into (cb_extrapolate_noalloc). `launched` is
+// set once the word has been cleared for a launch.
+struct CallerHistory {
+    const unsigned char* hist;
+    int* status;
+    bool launched;
+};
+
+// Zero a status word that every call shares, on the launch's stream.
+int clear_word(int* word, void* stream) {
+    cudaError_t e = cudaMemsetAsync(word, 0, sizeof(int), (cudaStream_t)stream);
+    return e == cudaSuccess ? CB_OK : cuda_fail(e, "cudaMemsetAsync");
+}
+
 // One skipped-step launch over the window `win` with the fp64 weights w[0..n).
 // With `feats` it is instead a full step's epilogue: a one-entry history (the
 // new features, weight 1) whose members are written, converted, into the ring
-// slot `next` while the hidden states receive x + sum_b g_b f_b.
+// slot `next` while the hidden states receive x + sum_b g_b f_b. With `ch` the
+// window's slots are read from ch->hist and events recorded in ch->status.
 int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs, cb_dtype out_dtype,
                void* const* resid, cb_dtype resid_dtype, void* stream, const void* const* gates = nullptr,
-               cb_dtype gate_dtype = CB_BF16, const void* const* feats = nullptr, cb_dtype feat_dtype = CB_BF16) {
-    if (!p->cache) return CB_ERR_UNBOUND;
+               cb_dtype gate_dtype = CB_BF16, const void* const* feats = nullptr, cb_dtype feat_dtype = CB_BF16,
+               CallerHistory* ch = nullptr) {
+    if (!ch && !p->cache) return CB_ERR_UNBOUND;
     const int K = win.n;
-    if (K < 1 || (!feats && p->count < K)) return CB_ERR_HISTORY_NOT_FULL;
+    if (K < 1 || (!feats && !ch && p->count < K)) return CB_ERR_HISTORY_NOT_FULL;
     if (!valid_dtype(out_dtype) || !valid_dtype(resid_dtype)) return CB_ERR_ARG;
     const int n = (int)p->tensors.size();
     const int ng = (int)p->groups.size();
@@ -315,7 +332,7 @@ int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs
     const bool cb16 = (feats ? feat_dtype : p->cache_dtype) == CB_BF16;
     const long long te = cbk::tile_elems(cb16);
     unsigned char* slot = p->cache + (size_t)p->next * p->slot_bytes;
-    A.hist_base = feats ? 0ull : (unsigned long long)(uintptr_t)p->cache;
+    A.hist_base = feats ? 0ull : (unsigned long long)(uintptr_t)(ch ? ch->hist : p->cache);
     A.copy_out = feats ? 1 : 0;
     for (int j = 0; j < CB_MAX_K; ++j) {
         const bool on = j < K;
@@ -387,7 +404,7 @@ int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs
     if (items == 0) return CB_OK;  // nothing requested
 
     A.wait_ns = p->wait_ns;
-    A.status = p->status_word();
+    A.status = ch ? ch->status : p->status_word();
     A.withhold_first = p->withhold_first;
     A.stages = 0;
     A.stage_chunks = K;
@@ -396,11 +413,17 @@ int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs
 
     rc = ensure_device(p);
     if (rc != CB_OK) return rc;
+    auto clear_status = [&]() {
+        if (!ch) return clear_status_once(p, stream);
+        const int r = clear_word(ch->status, stream);
+        ch->launched = r == CB_OK;
+        return r;
+    };
     auto launch_direct = [&]() {
         int grid = 0;
         int r = extrap_grid(p, K, cb16, (int)tiles, &grid);
         if (r != CB_OK) return r;
-        r = clear_status_once(p, stream);
+        r = clear_status();
         if (r != CB_OK) return r;
         cudaError_t e = any_gate ? cbk::launch_extrapolate_gated(A, K, cb16, grid, (cudaStream_t)stream)
                                  : cbk::launch_extrapolate(A, K, cb16, grid, (cudaStream_t)stream);
@@ -449,7 +472,7 @@ int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs
     if (cb16 && !grouped && K >= 3) frac = 0.75;
     const long long ctas = std::max(1LL, (long long)((double)p->dev.sms * per_sm * frac));
     const int grid = (int)(tiles < ctas ? tiles : ctas);
-    rc = clear_status_once(p, stream);
+    rc = clear_status();
     if (rc != CB_OK) return rc;
     cudaError_t e = any_gate ? cbk::launch_extrapolate_bulk_gated(A, K, cb16, grid, smem, (cudaStream_t)stream)
                              : cbk::launch_extrapolate_bulk(A, K, cb16, grouped, grid, smem, (cudaStream_t)stream);
@@ -642,6 +665,47 @@ int cb_extrapolate_ring(cb_plan* p, const double* slot_t, int head, double t_tar
     const int rc = weights_for(p, win, t_target, w);
     if (rc != CB_OK) return rc;
     return run_launch(p, win, w, outs, out_dtype, resid, resid_dtype, stream);
+}
+
+int cb_extrapolate_noalloc(cb_plan* p, const void* hist, size_t hist_bytes, const double* slot_t, int head,
+                           double t_target, void* const* outs, cb_dtype out_dtype, void* const* resid,
+                           cb_dtype resid_dtype, int* status, void* stream) {
+    if (!p || !hist || !slot_t || head < 0 || head >= p->K) return CB_ERR_ARG;
+    if (!aligned(hist, CB_CACHE_ALIGN)) return CB_ERR_ALIGN;
+    if (hist_bytes < p->slot_bytes * (size_t)p->K) return CB_ERR_ARG;  // the K slots, no status block
+    Window win{};
+    win.n = p->K;
+    for (int j = 0; j < p->K; ++j) {
+        win.slot[j] = (head + j) % p->K;
+        win.t[j] = slot_t[win.slot[j]];
+        if (!std::isfinite(win.t[j])) return CB_ERR_ARG;
+        win.tau[j] = p->tau(win.t[j]);
+        for (int i = 0; i < j; ++i)
+            if (win.t[i] == win.t[j]) return CB_ERR_NODES_DEGENERATE;
+    }
+    double w[CB_MAX_K];
+    int rc = weights_for(p, win, t_target, w);
+    if (rc != CB_OK) return rc;
+    // the library's status word on the current device (looked up on the first call there)
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (dev >= cbk::kMaxStatusDevices) return CB_ERR_LIMIT;
+    int* word = nullptr;
+    e = cbk::noalloc_status_word(dev, &word);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress");
+    CallerHistory ch{static_cast<const unsigned char*>(hist), word, false};
+    rc = run_launch(p, win, w, outs, out_dtype, resid, resid_dtype, stream, nullptr, CB_BF16, nullptr, CB_BF16, &ch);
+    if (rc != CB_OK) return rc;
+    if (status) {
+        if (!ch.launched) {  // nothing was requested, so nothing ran
+            *status = 0;
+            return CB_OK;
+        }
+        e = cudaMemcpyAsync(status, word, sizeof(int), cudaMemcpyDeviceToHost, (cudaStream_t)stream);
+        if (e != cudaSuccess) return cuda_fail(e, "status read-back");
+    }
+    return CB_OK;
 }
 
 int cb_extrapolate_weights(cb_plan* p, const double* w_logical, void* const* outs, cb_dtype out_dtype,
