@@ -28,11 +28,12 @@ namespace {
 
 constexpr float kU = 0x1.0p-24f;
 
-__device__ __forceinline__ uint4 ld_stream(const unsigned char* p) {
+// Plain 16-byte global load of history values (direct-load kernel). The
+// streaming form (ld.global.nc with L1::no_allocate) measured slower on GB300:
+// the FLUX skipped step took 2159 us with it and 1940 us without.
+__device__ __forceinline__ uint4 ld_v4(const unsigned char* p) {
     uint4 v;
-    asm("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
-        : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-        : "l"(p));
+    asm("ld.global.v4.u32 {%0,%1,%2,%3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
     return v;
 }
 

@@ -7,8 +7,8 @@
 //   * one persistent grid covers every tensor of every block; tiles of 4096
 //     (bf16) or 2048 (fp32) elements are dealt round-robin to the CTAs, and
 //     each CTA walks its item table forward, so no search is needed;
-//   * every thread issues all of its K x 16-B non-coherent, L1-bypassing loads
-//     (bf16: two 8-element vectors, fp32: one) before any arithmetic;
+//   * every thread issues all of its K x 16-B plain global loads (bf16: two
+//     8-element vectors, fp32: one) before any arithmetic;
 //   * the weights arrive as kernel parameters (fp32 high/low pairs).
 // The arithmetic is in cb_math.cuh. The bulk-copy pipeline variant
 // (bulk_kernel.cuh) computes the same bits from shared memory. GATED: the
@@ -30,8 +30,8 @@ __device__ __forceinline__ void load_member(const ExtrapArgs& A, long long moff,
 #pragma unroll
         for (int j = 0; j < K; ++j) {
             const unsigned char* p = hist_ptr(A, j, moff) + ev[u] * ES;
-            raw[u][j][0] = ld_stream(p);
-            if constexpr (!CB16) raw[u][j][CB16 ? 0 : 1] = ld_stream(p + 16);
+            raw[u][j][0] = ld_v4(p);
+            if constexpr (!CB16) raw[u][j][CB16 ? 0 : 1] = ld_v4(p + 16);
         }
 }
 

@@ -12,11 +12,12 @@
 namespace cbk {
 namespace {
 
-__device__ __forceinline__ uint4 ld_stream(const void* p) {
+// Plain 16-byte global load. The streaming form (ld.global.nc with
+// L1::no_allocate) measured 4.5 % slower on a 1:1 copy of the FLUX slot on
+// GB300 (663 against 635 us for 2 x 2.15 GB at 4 CTAs per SM).
+__device__ __forceinline__ uint4 ld_v4(const void* p) {
     uint4 v;
-    asm("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
-        : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-        : "l"(p));
+    asm("ld.global.v4.u32 {%0,%1,%2,%3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
     return v;
 }
 
@@ -34,11 +35,11 @@ template <bool SB>
 __device__ __forceinline__ Raw<SB> load8(const void* src, long long e) {
     Raw<SB> r;
     if constexpr (SB) {
-        r.w[0] = ld_stream(reinterpret_cast<const uint16_t*>(src) + e);
+        r.w[0] = ld_v4(reinterpret_cast<const uint16_t*>(src) + e);
     } else {
         const float* p = reinterpret_cast<const float*>(src) + e;
-        r.w[0] = ld_stream(p);
-        r.w[SB ? 0 : 1] = ld_stream(p + 4);
+        r.w[0] = ld_v4(p);
+        r.w[SB ? 0 : 1] = ld_v4(p + 4);
     }
     return r;
 }
