@@ -31,7 +31,7 @@ INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CFLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O2"]
 SOURCES = ["extrapolate.cu", "extrapolate_gated.cu", "extrapolate_bulk.cu", "extrapolate_bulk_gated.cu",
-           "push.cu", "static_status.cu", "plan.cpp"]
+           "push.cu", "epilogue.cu", "static_status.cu", "plan.cpp"]
 
 
 def _nvcc() -> str:

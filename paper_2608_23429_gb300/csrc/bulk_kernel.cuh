@@ -1,5 +1,7 @@
 // Skipped-step kernel, bulk-copy pipeline variant (same arithmetic and bits as
-// the direct kernel; Sec. 3.3, Eq. for f_t; Alg. 1, extrapolation branch).
+// the direct kernel on whole tiles; a tensor's ragged last tile takes the
+// compensated path for every element here. Sec. 3.3, Eq. for f_t; Alg. 1,
+// extrapolation branch).
 //
 // One or two CTAs per SM (see Shape). A producer lane moves,
 // for every work unit (one tile of one branch tensor), the K history chunks of
@@ -323,11 +325,10 @@ __global__ void __launch_bounds__(Shape<CB16, K, GROUPED, GATED>::threads, Shape
                             dot2_step(A.w_hi[j], A.w_lo[j], f, p, cc);
                         }
                         two_sum(p, cc, h, l);
-                        if constexpr (GATED) {
-                            (void)qq;
-                            const void* gm = A.m_gate[first + m];
-                            float gv = 1.0f;
-                            if (gm) gv = load_elem(A.stage_gate_bytes ? gate_stage(st) : gm, A.gate_bf16, gi[v] + e);
+                        // a member without a gate adds like an ungated one (as exact_resid)
+                        const void* gm = GATED ? A.m_gate[first + m] : nullptr;
+                        if (gm) {
+                            const float gv = load_elem(A.stage_gate_bytes ? gate_stage(st) : gm, A.gate_bf16, gi[v] + e);
                             add_gated_pair(gv, h, l, tp, tc);
                         } else {
                             two_sum(tp, h, tp, qq);

@@ -111,6 +111,13 @@ cudaError_t prepare_extrapolate_bulk_gated(int K, bool cache_bf16, size_t smem);
 cudaError_t launch_extrapolate_bulk_gated(const ExtrapArgs& a, int K, bool cache_bf16, int grid, size_t smem,
                                           cudaStream_t s);
 
+// Full-step epilogue kernel (epilogue.cu) for ungated bf16 features: a
+// one-entry history of weight 1 on 2048-element tiles, one 8-element vector
+// per thread and tile.
+constexpr long long epilogue_tile_elems = (long long)kThreads * kVecElems;
+cudaError_t launch_epilogue(const ExtrapArgs& a, int grid, cudaStream_t s);
+cudaError_t epilogue_blocks_per_sm(int* blocks);
+
 cudaError_t launch_push(const PushArgs& a, bool src_bf16, bool dst_bf16, int grid, cudaStream_t s);
 cudaError_t push_blocks_per_sm(bool src_bf16, bool dst_bf16, int* blocks);
 

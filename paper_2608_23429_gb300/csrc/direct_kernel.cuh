@@ -111,7 +111,8 @@ __device__ __forceinline__ void item_vectors(const ExtrapArgs& A, int it, const 
                 [&](int u, int e, float xe, float& hi, float& lo) {
                     exact_resid<CB16>(A, K, it, ev[u] + e, xe, hi, lo);
                 },
-                (K == 1 && A.copy_out) ? A.w_guard[0] : 1.0f);
+                // member_one's sums are unscaled (bf16 epilogue); member_fast's are scaled
+                (K == 1 && CB16 && A.copy_out) ? A.w_guard[0] : 1.0f);
     }
 }
 

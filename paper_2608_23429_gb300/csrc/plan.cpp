@@ -66,6 +66,7 @@ struct DeviceInfo {
     int smem_per_sm = 0;                   // shared memory of one SM
     int occ_extrap[2][CB_MAX_K + 1] = {};  // [cache_bf16][K]
     int occ_push[2][2] = {};               // [src_bf16][dst_bf16]
+    int occ_epilogue = 0;                  // epilogue kernel (bf16 features, no gates)
     int bulk_stages[2][CB_MAX_K + 1] = {};  // 1 once the kernel's shared-memory limit is raised
     int bulk_gated[2][CB_MAX_K + 1] = {};   // the same for the gated kernel
 };
@@ -330,7 +331,17 @@ int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs
     cbk::ExtrapArgs& A = *p->eargs;
     // the kernels' source type: the cache's, or the new features'
     const bool cb16 = (feats ? feat_dtype : p->cache_dtype) == CB_BF16;
-    const long long te = cbk::tile_elems(cb16);
+    // A full step's epilogue runs its own kernel (unless CB_OPT_KERNEL names
+    // one) when its threads keep enough loads in flight: ungated bf16 features
+    // with every tensor in a residual group of three or more branches.
+    // Otherwise the bulk pipeline streams faster (see epilogue.cu).
+    bool epilogue = feats && p->kernel == CB_KERNEL_AUTO && feat_dtype == CB_BF16 && resid;
+    for (int i = 0; epilogue && i < n; ++i) {
+        const int g = p->tensors[i].group;
+        epilogue = g >= 0 && resid[g] && p->groups[g].size() >= 3 && !(gates && gates[i]);
+    }
+    const long long te_bulk = cbk::tile_elems(cb16);
+    const long long te = epilogue ? cbk::epilogue_tile_elems : te_bulk;
     unsigned char* slot = p->cache + (size_t)p->next * p->slot_bytes;
     A.hist_base = feats ? 0ull : (unsigned long long)(uintptr_t)(ch ? ch->hist : p->cache);
     A.copy_out = feats ? 1 : 0;
@@ -430,6 +441,23 @@ int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs
         if (e != cudaSuccess) return cuda_fail(e, "extrapolate launch");
         return (int)CB_OK;
     };
+    if (epilogue) {
+        int& occ = p->dev.occ_epilogue;
+        if (occ == 0) {
+            cudaError_t e = cbk::epilogue_blocks_per_sm(&occ);
+            if (e != cudaSuccess || occ <= 0) {
+                occ = 0;
+                return cuda_fail(e == cudaSuccess ? cudaErrorInvalidConfiguration : e, "occupancy");
+            }
+        }
+        const long long ctas = (long long)p->dev.sms * occ;
+        const int grid = (int)(tiles < ctas ? tiles : ctas);
+        rc = clear_status();
+        if (rc != CB_OK) return rc;
+        cudaError_t e = cbk::launch_epilogue(A, grid, (cudaStream_t)stream);
+        if (e != cudaSuccess) return cuda_fail(e, "epilogue launch");
+        return CB_OK;
+    }
     if (p->kernel == CB_KERNEL_DIRECT) return launch_direct();
     // bf16 hidden states travel through shared memory with the last member of
     // their group; the pipeline must hold a whole group plus one stage ahead
@@ -449,7 +477,7 @@ int run_launch(cb_plan* p, const Window& win, const double* w, void* const* outs
             bool gated_item = false;
             for (int m = 0; m < A.nb[i]; ++m) gated_item = gated_item || A.m_gate[A.first[i] + m];
             if (!gated_item || !A.vec_ok[i]) continue;
-            fits = fits && (long long)A.i_row[i] >= te;
+            fits = fits && (long long)A.i_row[i] >= te_bulk;
             need = std::max(need, 2 * (size_t)A.i_hidden[i] * gs);
         }
         if (fits && need <= kMaxStagedGateBytes) A.stage_gate_bytes = (unsigned)((need + 127) / 128 * 128);

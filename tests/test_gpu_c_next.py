@@ -251,15 +251,17 @@ def test_gated_every_history_size(cb, H, K):
 
 @pytest.mark.parametrize("src", ["fp32", "bf16"])
 @pytest.mark.parametrize("odd", [False, True])
-def test_push_residual(cb, H, src, odd):
-    """Full step with the fused epilogue: the slots hold exactly what the plain
-    push writes, and x <- x + sum_b g_b f_b (un-rounded features) matches the
-    oracle's single rounding."""
+@pytest.mark.parametrize("kernel", ["auto", "bulk", "direct"])
+def test_push_residual(cb, H, src, odd, kernel):
+    """Full step with the fused epilogue (auto: its own kernel; bulk, direct:
+    the skipped-step kernels on a one-entry history): the slots hold exactly
+    what the plain push writes, and x <- x + sum_b g_b f_b (un-rounded
+    features) matches the oracle's single rounding."""
     from test_gpu_a_parity import _odd_workload
     w = _odd_workload(3) if odd else workloads.scaled(workloads.pixart(), 32)
     w.cache_dtype = "bf16"
     nodes = [900.0, 800.0, 700.0]
-    a = H.Walk(w, K=3, node_t=nodes)
+    a = H.Walk(w, K=3, node_t=nodes, kernel=kernel)
     b = H.Walk(w, K=3, node_t=nodes)
     cb.cb_plan_set_shapes(a.plan, [t.shape for t in w.tensors])
     tdt = torch.float32 if src == "fp32" else torch.bfloat16
@@ -291,6 +293,90 @@ def test_push_residual(cb, H, src, odd):
             assert st["exact"] >= 0.99 * st["n"], st  # compensated sum: rounded once, like the oracle
     a.close()
     b.close()
+
+
+@pytest.mark.parametrize("src", ["fp32", "bf16"])
+@pytest.mark.parametrize("gated", [False, True])
+def test_push_residual_kernels_bit_identical(cb, H, src, gated):
+    """The kernels that can run a full step's epilogue write the same slot
+    bytes and the same hidden-state bits (one shared arithmetic). Every tensor
+    sits in a group of three branches, so that with bf16 features and no gates
+    the default picks the epilogue kernel: whole tiles, ragged tiles (6006
+    elements) and a hidden state off the 16-byte grid (scalar path). In the
+    ragged last tile of a tensor the bulk kernel computes every element by the
+    compensated path while the others take the guarded fast path vector by
+    vector, so there the bulk kernel is held to the oracle's gate only."""
+    tensors = [workloads.TensorSpec(0, b, (2, 3, 1001), 0) for b in range(3)]
+    tensors += [workloads.TensorSpec(1, b, (2, 128, 1152), 1) for b in range(3)]
+    tensors += [workloads.TensorSpec(2, b, (1, 7, 64), 2) for b in range(3)]
+    w = workloads.Workload(name="groups-of-3", tensors=tensors, K=3, cache_dtype="bf16", T=0, r=0, t_min=0.0,
+                           t_max=999.0, timesteps=[], degree=6, noise=0.1, seed=55)
+    nodes = [900.0, 800.0, 700.0]
+    walks = {k: H.Walk(w, K=3, node_t=nodes, kernel=k) for k in ("auto", "bulk", "direct")}
+    for wk in walks.values():
+        cb.cb_plan_set_shapes(wk.plan, [t.shape for t in w.tensors])
+    tdt = torch.float32 if src == "fp32" else torch.bfloat16
+    ng = walks["auto"].n_groups
+    offs, slot = H.slot_layout([s_.numel for s_ in w.tensors], 2)
+    for k, t in enumerate(nodes):
+        feats = [workloads.trajectory(w, i, t, k, "cuda", out_dtype=tdt) for i in range(len(w.tensors))]
+        gates = _gates(w, torch.bfloat16, 40 + k, skip={1}) if gated else None
+        out = {}
+        for name, wk in walks.items():
+            resid = [workloads.hidden_state(w, g, "cuda", salt=k) for g in range(ng)]
+            x2 = resid[2].reshape(-1)
+            shifted = torch.empty(x2.numel() + 1, dtype=x2.dtype, device="cuda")[1:]  # 2 bytes off the grid
+            shifted.copy_(x2)
+            resid[2] = shifted
+            cb.cb_cache_push_residual(wk.plan, feats, H.CB[src], t, resid, cb.CB_BF16, gates, cb.CB_BF16)
+            torch.cuda.synchronize()
+            assert cb.cb_plan_device_status(wk.plan) == 0
+            out[name] = resid
+        # the default runs the epilogue kernel for ungated bf16 features, else the bulk kernel
+        ran = {"auto": "epilogue" if src == "bf16" and not gated else "bulk", "bulk": "bulk", "direct": "direct"}
+        for name in ("bulk", "direct"):
+            for i, s_ in enumerate(w.tensors):  # the slot just written (padding and other slots are not)
+                lo = k * slot + offs[i]
+                assert torch.equal(walks["auto"].cache[lo:lo + 2 * s_.numel], walks[name].cache[lo:lo + 2 * s_.numel]), \
+                    (k, name, i)
+            for g in range(ng):
+                a_, b_ = out["auto"][g].reshape(-1).view(torch.int16), out[name][g].reshape(-1).view(torch.int16)
+                if (ran["auto"] == "bulk") != (ran[name] == "bulk"):  # the bulk kernel's whole tiles only
+                    te = 4096 if src == "bf16" else 2048
+                    whole = a_.numel() // te * te
+                    a_, b_ = a_[:whole], b_[:whole]
+                assert torch.equal(a_, b_), (k, name, g)
+            # the bulk kernel's hidden states, whole and ragged tiles, against the oracle
+            for g in range(ng):
+                members = [i for i, s_ in enumerate(w.tensors) if s_.group == g]
+                F = [[H.host(feats[i])] for i in members]
+                G = None if gates is None else [None if gates[i] is None else H.expand_gate(gates[i],
+                                                                                            w.tensors[i].shape)
+                                                for i in members]
+                x0 = H.host(workloads.hidden_state(w, g, "cuda", salt=k))
+                _, r64 = orc.extrapolate(F, [1.0], H.ORC[src], None, X=x0, x_dtype=orc.BF16, resid_dtype=orc.FP64,
+                                         G=G)
+                Fd = np.array([f[0].astype(np.float64) if src == "fp32" else H.bf16_to_f64(f[0]) for f in F])
+                gb = np.array([np.ones_like(Fd[0]) if (G is None or x is None) else np.abs(x)
+                               for x in (G or [None] * 3)])
+                bound = (gb * np.abs(Fd)).sum(0) + np.abs(H.bf16_to_f64(x0))
+                st = H.compare_bf16(H.host(out[name][g]), orc.convert(r64, orc.FP64, orc.BF16), r64, bound)
+                assert st["bad"] == 0, (k, name, g, st)
+        # and against the oracle's single rounding
+        for g in range(ng):
+            members = [i for i, s_ in enumerate(w.tensors) if s_.group == g]
+            F = [[H.host(feats[i])] for i in members]
+            G = None if gates is None else [None if gates[i] is None else H.expand_gate(gates[i], w.tensors[i].shape)
+                                            for i in members]
+            x0 = H.host(workloads.hidden_state(w, g, "cuda", salt=k))
+            _, r64 = orc.extrapolate(F, [1.0], H.ORC[src], None, X=x0, x_dtype=orc.BF16, resid_dtype=orc.FP64, G=G)
+            Fd = np.array([f[0].astype(np.float64) if src == "fp32" else H.bf16_to_f64(f[0]) for f in F])
+            gb = np.array([np.ones_like(Fd[0]) if (G is None or x is None) else np.abs(x) for x in (G or [None] * 3)])
+            bound = (gb * np.abs(Fd)).sum(0) + np.abs(H.bf16_to_f64(x0))
+            st = H.compare_bf16(H.host(out["auto"][g]), orc.convert(r64, orc.FP64, orc.BF16), r64, bound)
+            assert st["bad"] == 0, (k, g, st)
+    for wk in walks.values():
+        wk.close()
 
 
 @pytest.mark.parametrize("layout", ["lone", "groups"])
