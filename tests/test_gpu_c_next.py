@@ -379,6 +379,52 @@ def test_push_residual_kernels_bit_identical(cb, H, src, gated):
         wk.close()
 
 
+@pytest.mark.parametrize("src", ["fp32", "bf16"])
+@pytest.mark.parametrize("kernel", ["auto", "bulk", "direct"])
+def test_push_residual_cancellation(cb, H, src, kernel):
+    """Full-step epilogue where the hidden-state update cancels. Group 0: the
+    first member's features are -x plus a residue, so x + sum_b f_b is a
+    residue of the terms. Group 1: a small hidden state (~1e-6) and members a,
+    b, -(a + b) + residue, which cancel among themselves (the fp32 sum a + b
+    is rounded, so the fast path is off by many bf16 ulps, and only the
+    members' part of the guard can see it). Every element must still be
+    within one ulp of the oracle."""
+    tensors = [workloads.TensorSpec(g, b, (2, 64, 1152), g) for g in range(2) for b in range(3)]
+    w = workloads.Workload(name="cancel", tensors=tensors, K=2, cache_dtype="bf16", T=0, r=0, t_min=0.0,
+                           t_max=999.0, timesteps=[], degree=6, noise=0.1, seed=57)
+    walk = H.Walk(w, K=2, node_t=[900.0, 800.0], kernel=kernel)
+    ng = walk.n_groups
+    gen = torch.Generator(device="cuda").manual_seed(5)
+    tdt = torch.float32 if src == "fp32" else torch.bfloat16
+    small = 1e-6 if src == "fp32" else 1e-3  # a bf16 residue cannot be smaller than ~ulp(x)
+    shape = w.tensors[0].shape
+    resid = [workloads.hidden_state(w, 0, "cuda"),
+             (1e-6 * torch.randn(shape, generator=gen, device="cuda")).to(torch.bfloat16)]
+    rh = [H.host(r) for r in resid]
+    x0 = resid[0].float()
+    a = torch.randn(shape, generator=gen, device="cuda").to(tdt).float()
+    b = torch.randn(shape, generator=gen, device="cuda").to(tdt).float()
+    feats = [-x0 + small * torch.randn(shape, generator=gen, device="cuda"),
+             small * torch.randn(shape, generator=gen, device="cuda"),
+             small * torch.randn(shape, generator=gen, device="cuda"),
+             a, b, -(a.double() + b.double()).float() + small * torch.randn(shape, generator=gen, device="cuda")]
+    feats = [f.to(tdt) for f in feats]
+    cb.cb_cache_push_residual(walk.plan, feats, H.CB[src], 900.0, resid, cb.CB_BF16)
+    torch.cuda.synchronize()
+    assert cb.cb_plan_device_status(walk.plan) == 0
+    for g in range(ng):
+        members = [i for i, s_ in enumerate(w.tensors) if s_.group == g]
+        F = [[H.host(feats[i])] for i in members]
+        _, r64 = orc.extrapolate(F, [1.0], H.ORC[src], None, X=rh[g], x_dtype=orc.BF16, resid_dtype=orc.FP64)
+        Fd = np.array([f[0].astype(np.float64) if src == "fp32" else H.bf16_to_f64(f[0]) for f in F])
+        bound = np.abs(Fd).sum(0) + np.abs(H.bf16_to_f64(rh[g]))
+        st = H.compare_bf16(H.host(resid[g]), orc.convert(r64, orc.FP64, orc.BF16), r64, bound)
+        assert st["bad"] == 0, (g, st)
+        if src == "fp32":  # the case is what it claims: the update cancels for most elements
+            assert np.median(np.abs(r64) / bound) < 1e-4, g
+    walk.close()
+
+
 @pytest.mark.parametrize("layout", ["lone", "groups"])
 def test_maximum_plan(cb, H, layout):
     """A plan at the ABI's limits: CB_MAX_TENSORS tensors and CB_MAX_K history
