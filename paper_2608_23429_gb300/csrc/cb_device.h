@@ -1,5 +1,6 @@
 // Internal: kernel argument blocks and launchers shared by the host plan
-// (plan.cpp) and the kernels (extrapolate*.cu, push.cu). Not part of the ABI.
+// (plan.cpp) and the kernels (extrapolate*.cu, epilogue.cu, push.cu), and the
+// library's own status block (static_status.cu). Not part of the ABI.
 #pragma once
 
 #include <cuda_runtime.h>

@@ -2,8 +2,8 @@
 // Sec. 3.3; Alg. 1 offline stage), the history buffer's ring bookkeeping, the
 // online weights (Sec. 3.2 Eq. barycentric_coeff) and the kernel launches.
 // Everything here is fp64 host arithmetic that runs in microseconds per call;
-// all device work is in push.cu and the extrapolate*.cu instantiations of the
-// skipped-step kernels.
+// all device work is in push.cu (cache write), epilogue.cu (full-step
+// epilogue) and the extrapolate*.cu instantiations of the skipped-step kernels.
 #include <cuda_runtime.h>
 
 #include <algorithm>
