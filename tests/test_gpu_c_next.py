@@ -297,18 +297,24 @@ def test_push_residual(cb, H, src, odd, kernel):
 
 @pytest.mark.parametrize("src", ["fp32", "bf16"])
 @pytest.mark.parametrize("gated", [False, True])
-def test_push_residual_kernels_bit_identical(cb, H, src, gated):
+@pytest.mark.parametrize("layout", ["groups-of-3", "pairs"])
+def test_push_residual_kernels_bit_identical(cb, H, src, gated, layout):
     """The kernels that can run a full step's epilogue write the same slot
     bytes and the same hidden-state bits (one shared arithmetic). Every tensor
-    sits in a group of three branches, so that with bf16 features and no gates
-    the default picks the epilogue kernel: whole tiles, ragged tiles (6006
-    elements) and a hidden state off the 16-byte grid (scalar path). In the
+    sits in a group of three branches (with bf16 features and no gates the
+    default then picks the epilogue kernel), or every item has one or two
+    (groups of two and lone tensors: the bulk kernel): whole tiles, ragged
+    tiles (6006 elements) and a hidden state off the 16-byte grid (scalar
+    path). In the
     ragged last tile of a tensor the bulk kernel computes every element by the
     compensated path while the others take the guarded fast path vector by
     vector, so there the bulk kernel is held to the oracle's gate only."""
-    tensors = [workloads.TensorSpec(0, b, (2, 3, 1001), 0) for b in range(3)]
-    tensors += [workloads.TensorSpec(1, b, (2, 128, 1152), 1) for b in range(3)]
-    tensors += [workloads.TensorSpec(2, b, (1, 7, 64), 2) for b in range(3)]
+    nbr = 3 if layout == "groups-of-3" else 2
+    tensors = [workloads.TensorSpec(0, b, (2, 3, 1001), 0) for b in range(nbr)]
+    tensors += [workloads.TensorSpec(1, b, (2, 128, 1152), 1) for b in range(nbr)]
+    tensors += [workloads.TensorSpec(2, b, (1, 7, 64), 2) for b in range(nbr)]
+    if layout == "pairs":  # lone tensors: items of one member without a hidden state
+        tensors += [workloads.TensorSpec(3 + i, 0, (1, 1, n), -1) for i, n in enumerate([1, 4097, 40000])]
     w = workloads.Workload(name="groups-of-3", tensors=tensors, K=3, cache_dtype="bf16", T=0, r=0, t_min=0.0,
                            t_max=999.0, timesteps=[], degree=6, noise=0.1, seed=55)
     nodes = [900.0, 800.0, 700.0]
@@ -332,8 +338,9 @@ def test_push_residual_kernels_bit_identical(cb, H, src, gated):
             torch.cuda.synchronize()
             assert cb.cb_plan_device_status(wk.plan) == 0
             out[name] = resid
-        # the default runs the epilogue kernel for ungated bf16 features, else the bulk kernel
-        ran = {"auto": "epilogue" if src == "bf16" and not gated else "bulk", "bulk": "bulk", "direct": "direct"}
+        # the default runs the epilogue kernel for ungated bf16 features in groups of three, else the bulk kernel
+        epi = src == "bf16" and not gated and layout == "groups-of-3"
+        ran = {"auto": "epilogue" if epi else "bulk", "bulk": "bulk", "direct": "direct"}
         for name in ("bulk", "direct"):
             for i, s_ in enumerate(w.tensors):  # the slot just written (padding and other slots are not)
                 lo = k * slot + offs[i]
@@ -358,7 +365,7 @@ def test_push_residual_kernels_bit_identical(cb, H, src, gated):
                                          G=G)
                 Fd = np.array([f[0].astype(np.float64) if src == "fp32" else H.bf16_to_f64(f[0]) for f in F])
                 gb = np.array([np.ones_like(Fd[0]) if (G is None or x is None) else np.abs(x)
-                               for x in (G or [None] * 3)])
+                               for x in (G or [None] * len(members))])
                 bound = (gb * np.abs(Fd)).sum(0) + np.abs(H.bf16_to_f64(x0))
                 st = H.compare_bf16(H.host(out[name][g]), orc.convert(r64, orc.FP64, orc.BF16), r64, bound)
                 assert st["bad"] == 0, (k, name, g, st)
@@ -371,7 +378,8 @@ def test_push_residual_kernels_bit_identical(cb, H, src, gated):
             x0 = H.host(workloads.hidden_state(w, g, "cuda", salt=k))
             _, r64 = orc.extrapolate(F, [1.0], H.ORC[src], None, X=x0, x_dtype=orc.BF16, resid_dtype=orc.FP64, G=G)
             Fd = np.array([f[0].astype(np.float64) if src == "fp32" else H.bf16_to_f64(f[0]) for f in F])
-            gb = np.array([np.ones_like(Fd[0]) if (G is None or x is None) else np.abs(x) for x in (G or [None] * 3)])
+            gb = np.array([np.ones_like(Fd[0]) if (G is None or x is None) else np.abs(x)
+                           for x in (G or [None] * len(members))])
             bound = (gb * np.abs(Fd)).sum(0) + np.abs(H.bf16_to_f64(x0))
             st = H.compare_bf16(H.host(out["auto"][g]), orc.convert(r64, orc.FP64, orc.BF16), r64, bound)
             assert st["bad"] == 0, (k, g, st)
@@ -381,15 +389,18 @@ def test_push_residual_kernels_bit_identical(cb, H, src, gated):
 
 @pytest.mark.parametrize("src", ["fp32", "bf16"])
 @pytest.mark.parametrize("kernel", ["auto", "bulk", "direct"])
-def test_push_residual_cancellation(cb, H, src, kernel):
+@pytest.mark.parametrize("layout", ["groups-of-3", "pairs"])
+def test_push_residual_cancellation(cb, H, src, kernel, layout):
     """Full-step epilogue where the hidden-state update cancels. Group 0: the
     first member's features are -x plus a residue, so x + sum_b f_b is a
     residue of the terms. Group 1: a small hidden state (~1e-6) and members a,
     b, -(a + b) + residue, which cancel among themselves (the fp32 sum a + b
     is rounded, so the fast path is off by many bf16 ulps, and only the
-    members' part of the guard can see it). Every element must still be
-    within one ulp of the oracle."""
-    tensors = [workloads.TensorSpec(g, b, (2, 64, 1152), g) for g in range(2) for b in range(3)]
+    members' part of the guard can see it). With pairs (groups of two) the
+    members are -x + residue and a residue, then a and -a + residue. Every
+    element must still be within one ulp of the oracle."""
+    nbr = 3 if layout == "groups-of-3" else 2
+    tensors = [workloads.TensorSpec(g, b, (2, 64, 1152), g) for g in range(2) for b in range(nbr)]
     w = workloads.Workload(name="cancel", tensors=tensors, K=2, cache_dtype="bf16", T=0, r=0, t_min=0.0,
                            t_max=999.0, timesteps=[], degree=6, noise=0.1, seed=57)
     walk = H.Walk(w, K=2, node_t=[900.0, 800.0], kernel=kernel)
@@ -404,10 +415,12 @@ def test_push_residual_cancellation(cb, H, src, kernel):
     x0 = resid[0].float()
     a = torch.randn(shape, generator=gen, device="cuda").to(tdt).float()
     b = torch.randn(shape, generator=gen, device="cuda").to(tdt).float()
-    feats = [-x0 + small * torch.randn(shape, generator=gen, device="cuda"),
-             small * torch.randn(shape, generator=gen, device="cuda"),
-             small * torch.randn(shape, generator=gen, device="cuda"),
-             a, b, -(a.double() + b.double()).float() + small * torch.randn(shape, generator=gen, device="cuda")]
+    def residue():
+        return small * torch.randn(shape, generator=gen, device="cuda")
+    if nbr == 3:
+        feats = [-x0 + residue(), residue(), residue(), a, b, -(a.double() + b.double()).float() + residue()]
+    else:
+        feats = [-x0 + residue(), residue(), a, -a + residue()]
     feats = [f.to(tdt) for f in feats]
     cb.cb_cache_push_residual(walk.plan, feats, H.CB[src], 900.0, resid, cb.CB_BF16)
     torch.cuda.synchronize()
