@@ -34,13 +34,20 @@ sys.path.insert(0, ROOT)
 
 METRIC = "extrapolation GB/s & % of HBM peak; µs per skipped step (all blocks), 1 GB300"
 # configurations timed after the headline (FLUX.1-dev 1024^2), each on its own
-# filled history: (preset, [(variant, hidden states fused)])
+# filled history: (preset, [(variant, step, hidden states fused, gated)]).
+# step "skip" is a skipped step (cb_extrapolate / cb_extrapolate_gated);
+# "full" a full step's cache write (cb_cache_push) and "full-fused" the cache
+# write with the hidden-state update (cb_cache_push_residual); full steps run
+# after the skipped ones, from an emptied history.
 OTHER_WORKLOADS = [
-    ("pixart", [("prediction-only", False), ("fused", True)]),
-    ("dit512", [("prediction-only", False)]),
-    ("dit256", [("fused", True), ("prediction-only", False)]),
-    ("dit256-k3", [("fused", True), ("prediction-only", False)]),
-    ("flux", [("fused", True)]),
+    ("pixart", [("prediction-only", "skip", False, False), ("fused", "skip", True, False),
+                ("gated", "skip", True, True), ("full-step epilogue", "full-fused", True, False)]),
+    ("dit512", [("prediction-only", "skip", False, False)]),
+    ("dit256", [("fused", "skip", True, False), ("prediction-only", "skip", False, False),
+                ("gated", "skip", True, True), ("full-step epilogue, gated", "full-fused", True, True)]),
+    ("dit256-k3", [("fused", "skip", True, False), ("prediction-only", "skip", False, False)]),
+    ("flux", [("fused", "skip", True, False), ("cache write", "full", False, False),
+              ("full-step epilogue", "full-fused", True, False)]),
 ]
 NOMINAL_HBM_GBS = 7900.0
 KERNEL_SOURCES = ["paper_2608_23429_gb300/csrc/extrapolate_bulk.cu", "paper_2608_23429_gb300/csrc/bulk_kernel.cuh",
@@ -276,9 +283,10 @@ def fill_window(torch, cb, wl, w, plan, cdt, pushed, dev, stream):
 
 
 def time_workload(torch, cb, wl, dev, name: str, variants, steps: int, warmup: int, peak: float) -> list:
-    """Skipped steps of one more workload in the launch configuration of the
+    """More steps of one more workload in the launch configuration of the
     headline: the same window walk, one launch per step, per-launch events on
-    the launching stream. variants: (label, fused) pairs on one filled history."""
+    the launching stream. variants: (label, step, fused, gated) on one filled
+    history (see OTHER_WORKLOADS)."""
     w = wl.PRESETS[name]()
     K = w.K
     pushed, targets = pick_window(w, cb)
@@ -287,6 +295,7 @@ def time_workload(torch, cb, wl, dev, name: str, variants, steps: int, warmup: i
     tdt = torch.bfloat16 if w.cache_dtype == "bf16" else torch.float32
     plan = cb.cb_plan_create(node_t, K, [(t.layer, t.branch, t.numel, t.group) for t in w.tensors], cdt,
                              w.t_min, w.t_max)
+    cb.cb_plan_set_shapes(plan, [t.shape for t in w.tensors])
     cache = torch.empty(cb.cb_plan_cache_bytes(plan), dtype=torch.uint8, device=dev)
     cb.cb_plan_bind_cache(plan, cache, cache.numel())
     stream = torch.cuda.Stream(device=dev)
@@ -296,17 +305,54 @@ def time_workload(torch, cb, wl, dev, name: str, variants, steps: int, warmup: i
     slot_elems = sum(t.numel for t in w.tensors)
     esz = 2 if w.cache_dtype == "bf16" else 4
     t_targets = [w.timesteps[s] for s in targets]
+    gg = torch.Generator(device=dev).manual_seed(7)
+    gates = [(0.5 * torch.randn(t.shape[0], t.shape[-1], generator=gg, device=dev)).to(torch.bfloat16)
+             for t in w.tensors]
+    gate_bytes = sum(t.shape[0] * t.shape[-1] * 2 for t in w.tensors)
+    src = None
+    # fresh, strictly monotone times for the full steps (pushed from an emptied history)
+    span = (w.timesteps[-1] - w.timesteps[0]) / 1e6
+    push_t = iter([w.timesteps[0] + span * i for i in range(1000000)])
     rows = []
-    for label, fused in variants:
+    for label, step, fused, gated in variants:
         resid = [wl.hidden_state(w, g, dev) for g in range(n_groups)] if fused else None
         resid_elems = sum(w.group_numel(g) for g in range(n_groups)) if fused else 0
-        bytes_step = slot_elems * esz * (K + 1) + resid_elems * 2 * 2
         outs_p = cb.ptr_array(outs)
         resid_p = cb.ptr_array(resid) if resid is not None else None
+        gates_p = cb.ptr_array(gates) if gated else None
+        if step == "skip":
+            # K slot reads + one output write (+ hidden state read and write, + gates)
+            bytes_step = slot_elems * esz * (K + 1) + resid_elems * 2 * 2 + (gate_bytes if gated else 0)
+
+            def launch(k):
+                t = t_targets[k % len(t_targets)]
+                if gated:
+                    cb.cb_extrapolate_gated(plan, t, outs_p, cdt, resid_p, cb.CB_BF16, gates_p, cb.CB_BF16,
+                                            stream=stream)
+                else:
+                    cb.cb_extrapolate(plan, t, outs_p, cdt, resid_p, cb.CB_BF16, stream=stream)
+        else:
+            if src is None:  # the features of one generated full step, re-pushed with fresh times
+                src = [wl.trajectory(w, i, w.timesteps[pushed[-1]], pushed[-1], dev) for i in range(len(w.tensors))]
+                torch.cuda.synchronize()
+                cb.cb_plan_reset(plan)
+            src_p = cb.ptr_array(src)
+            # features read + slot written (+ hidden state read and write, + gates)
+            bytes_step = slot_elems * (src[0].element_size() + esz)
+            if step == "full-fused":
+                bytes_step += resid_elems * 2 * 2 + (gate_bytes if gated else 0)
+
+            def launch(k):
+                t = next(push_t)
+                if step == "full":
+                    cb.cb_cache_push(plan, src_p, cdt, t, stream=stream)
+                else:
+                    cb.cb_cache_push_residual(plan, src_p, cdt, t, resid_p, cb.CB_BF16, gates_p, cb.CB_BF16,
+                                              stream=stream)
         w0, w1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         w0.record(stream)
         for k in range(warmup):
-            cb.cb_extrapolate(plan, t_targets[k % len(t_targets)], outs_p, cdt, resid_p, cb.CB_BF16, stream=stream)
+            launch(k)
         w1.record(stream)
         stream.synchronize()
         # at least ~0.3 s of timed steps, so that the clock sampler sees the load
@@ -315,8 +361,7 @@ def time_workload(torch, cb, wl, dev, name: str, variants, steps: int, warmup: i
         with Clocks(torch.cuda.current_device()) as clk:
             for k in range(n):
                 ev[k][0].record(stream)
-                cb.cb_extrapolate(plan, t_targets[k % len(t_targets)], outs_p, cdt, resid_p, cb.CB_BF16,
-                                  stream=stream)
+                launch(k)
                 ev[k][1].record(stream)
             stream.synchronize()
         clocks = clk.summary()
@@ -324,15 +369,15 @@ def time_workload(torch, cb, wl, dev, name: str, variants, steps: int, warmup: i
             raise RuntimeError(f"device status set while timing {name}")
         us = sorted(a.elapsed_time(b) * 1e3 for a, b in ev)
         mean_us = sum(us) / len(us)
-        rows.append({"workload": w.name, "variant": label, "K": K, "fused_residual": bool(fused),
-                     "bytes_per_step": bytes_step, "us_per_step": round(mean_us, 2),
+        rows.append({"workload": w.name, "variant": label, "step": step, "K": K, "fused_residual": bool(fused),
+                     "gated": bool(gated), "bytes_per_step": bytes_step, "us_per_step": round(mean_us, 2),
                      "us_per_step_median": round(us[len(us) // 2], 2),
                      "gbs": round(bytes_step / (mean_us * 1e-6) / 1e9, 2),
                      "frac": round(bytes_step / (mean_us * 1e-6) / 1e9 / peak, 4), "steps": n,
                      "clocks": {"sm_mhz": clocks["sm_mhz"], "reasons": clocks["reasons"]}})
         del resid
     cb.cb_plan_destroy(plan)
-    del cache, outs
+    del cache, outs, src
     torch.cuda.empty_cache()
     return rows
 
