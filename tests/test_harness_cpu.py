@@ -87,3 +87,28 @@ def test_merge_adds_counts_and_keeps_maxima(H):
     b = dict(n=5, exact=3, one_ulp=1, floor=1, bad=0, max_ulp=9)
     m = H.merge([a, b])
     assert m == dict(n=15, exact=11, one_ulp=3, floor=1, bad=0, max_ulp=9)
+
+
+def test_bench_parity_record_agrees_with_the_harness(H):
+    """bench.py's parity record (the timed FLUX step against the oracle)
+    counts exactly as the GPU tests' gate: the same ulp distances, the same
+    cancellation floor, on patterns 0..3 values apart and on cancellations
+    inside and outside the floor."""
+    import bench
+    rng = np.random.default_rng(11)
+    ref, ref64 = _ref(H, rng.standard_normal(3000) * 10.0 ** rng.integers(-20, 20, 3000))
+    bound = np.abs(ref64)
+    gpu = ref.copy()
+    gpu[:600] = H._step(ref[:600], 1)
+    gpu[600:900] = H._step(ref[600:900], -2)
+    gpu[900:1000] = H._step(ref[900:1000], 3)
+    # exact value ~0 beside large terms: a gpu value within the floor passes, one outside fails
+    ref64[1000:1100] = 0.0
+    ref[1000:1100] = 0
+    bound[1000:1100] = 2.0 ** 50
+    gpu[1000:1050] = H.orc.bf16_encode(np.full(50, 2.0 ** 9))    # 2^9 <= 2^-40 * 2^50: inside the floor
+    gpu[1050:1100] = H.orc.bf16_encode(np.full(50, 2.0 ** 11))   # outside it
+    mine = bench.parity_stats(gpu, ref, ref64, bound)
+    theirs = H.compare_bf16(gpu, ref, ref64, bound)
+    assert mine == theirs
+    assert mine["one_ulp"] == 600 and mine["floor"] == 50 and mine["bad"] == 300 + 100 + 50
