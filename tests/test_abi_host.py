@@ -160,6 +160,38 @@ def test_validation_before_launch(cb):
     cb.cb_plan_destroy(p)
 
 
+def test_noalloc_validation_before_any_cuda_call(cb):
+    """cb_extrapolate_noalloc checks its arguments before it touches CUDA (its
+    per-device set-up included), so every malformed call below returns its
+    code on a machine without a GPU. The plan is never bound: the call needs
+    no arena."""
+    p = cb.cb_plan_create([999.0, 900.0, 800.0], 3, _tensors([64, 64], [0, 0]), cb.CB_BF16, 0.0, 999.0)
+    st = cb.raw_status
+    arr = lambda *xs: (ctypes.c_void_p * len(xs))(*xs)
+    need = cb.cb_plan_cache_bytes(p) - cb.CB_STATUS_BYTES  # the K slots, no status block
+    times = (ctypes.c_double * 3)(999.0, 900.0, 800.0)
+    outs = arr(0x1000, 0x2000)
+    hist = 0x100000  # never dereferenced below
+    call = lambda h, nbytes, t, head, tgt, o=outs: st("cb_extrapolate_noalloc", p, h, nbytes, t, head, tgt, o, 0,
+                                                      None, 0, None, None)
+    assert call(None, need, times, 0, 850.0) == cb.CB_ERR_ARG            # no history buffer
+    assert call(hist + 16, need, times, 0, 850.0) == cb.CB_ERR_ALIGN     # not CB_CACHE_ALIGN-aligned
+    assert call(hist, need - 1, times, 0, 850.0) == cb.CB_ERR_ARG        # shorter than the K slots
+    assert call(hist, need, None, 0, 850.0) == cb.CB_ERR_ARG             # no slot times
+    assert call(hist, need, times, 3, 850.0) == cb.CB_ERR_ARG            # head outside [0, K)
+    assert call(hist, need, times, -1, 850.0) == cb.CB_ERR_ARG
+    assert call(hist, need, times, 0, float("nan")) == cb.CB_ERR_ARG     # target not finite
+    dup = (ctypes.c_double * 3)(999.0, 900.0, 999.0)
+    assert call(hist, need, dup, 0, 850.0) == cb.CB_ERR_NODES_DEGENERATE
+    bad = (ctypes.c_double * 3)(999.0, float("inf"), 800.0)
+    assert call(hist, need, bad, 0, 850.0) == cb.CB_ERR_ARG
+    assert st("cb_extrapolate_noalloc", None, hist, need, times, 0, 850.0, outs, 0, None, 0, None,
+              None) == cb.CB_ERR_ARG                                    # no plan
+    # the plan's own history is untouched, and it was never bound
+    assert cb.cb_plan_history(p, 3)[1:] == (0, 0)
+    cb.cb_plan_destroy(p)
+
+
 def test_failed_launch_leaves_history_unchanged(cb):
     torch = pytest.importorskip("torch")
     if torch.cuda.is_available():
