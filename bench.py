@@ -16,6 +16,16 @@ Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME]
                        [--impl ours|reference]
 Under torchrun each rank runs its own replica (independent samples, no data
 exchange); timing is the max over ranks.
+
+Besides the contract's keys, the JSON line carries: `roofline` (achieved GB/s
+of the timed kernel against the measured copy peak, DRAM traffic per launch
+from the committed ncu record when it matches the kernel sources),
+`schedule_loop` (Alg. 1's whole online stage over the schedule), `parity` (the
+timed step's predictions against the oracle on a sample), `workloads` (the
+other configurations and the gated, cache-write and full-step-epilogue paths,
+each with its own clock sample), `cpu_baseline` (the oracle on the host
+cores), `e2e` (the step through the public API from and to pinned host
+buffers) and `clocks`.
 """
 from __future__ import annotations
 

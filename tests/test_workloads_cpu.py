@@ -5,6 +5,7 @@ full/skipped step counts, and the statistical structure of the generated
 trajectories: a Chebyshev series of the stated degree whose d-th coefficient
 has standard deviation 1/(d+1)^2, additive N(0, 0.1^2) noise per node, and
 (DiT-XL/2 512^2) per-channel LogNormal(0, 1) scales. Same seed, same bytes.
+Also the window of each schedule that bench.py times.
 """
 import numpy as np
 import pytest
@@ -95,3 +96,19 @@ def test_noise_and_channel_scales():
 def _no_scale(w):
     w.lognormal = False
     return w
+
+
+@pytest.mark.parametrize("name", ["dit256", "dit256-k3", "dit512", "pixart", "flux"])
+def test_bench_timed_window(name):
+    """The window bench.py times: the full steps pushed before it end with K
+    equispaced full steps one refresh interval apart, past the warm-up, and
+    the targets are the skipped steps right after the last of them."""
+    import bench
+    w = wl.PRESETS[name]()
+    mask = orc.full_schedule(w.T, w.r, w.s0, w.s1, w.K)
+    pushed, targets = bench.window_of(w, mask)
+    win = pushed[-w.K:]
+    assert len(set(b - a for a, b in zip(win, win[1:]))) == 1 and win[-1] - win[0] == w.r * (w.K - 1)
+    assert all(mask[s] for s in pushed) and not any(mask[s] for s in targets)
+    assert targets == list(range(win[-1] + 1, targets[-1] + 1)) and mask[targets[-1] + 1]
+    assert pushed == [s for s in range(win[-1] + 1) if mask[s]]  # every full step up to the window, in order
